@@ -1,0 +1,1306 @@
+// C ABI: context, paged pool tables, per-call planning and launches.
+//
+// Host-side model of the paper's GPU state S_t = (R_t, Q_t) (Sec. III):
+//   * agents  -> registered prefixes of length ell_a; resident ones hold a
+//     run of pool pages (the prefix is paid once per agent, Eq. 2);
+//   * requests -> open requests of an agent with a private suffix page run;
+//   * the free-page list is the remaining budget B_t; a call that needs
+//     more pages than are free fails with TPA_ERR_NO_SPACE.
+// Every device-facing call builds one plan blob (page lists and work items)
+// in a pinned staging slot, uploads it with one copy and launches the
+// kernels.  Pages freed while queued work may still read them carry the
+// sequence number of that work; whoever reuses them first waits for it.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstddef>
+#include <cstdlib>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <unordered_map>
+#include <vector>
+
+#include "../../include/topas_attn.h"
+#include "kernels.h"
+
+namespace tpa {
+cudaError_t init_dense_kernels();
+cudaError_t init_suffix_kernels();
+}  // namespace tpa
+
+using namespace tpa;
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+#define CUDA_TRY(expr)                                                              \
+  do {                                                                              \
+    cudaError_t e_ = (expr);                                                        \
+    if (e_ != cudaSuccess)                                                          \
+      return fail(TPA_ERR_CUDA, "%s: %s (%s:%d)", #expr, cudaGetErrorString(e_),    \
+                  __FILE__, __LINE__);                                              \
+  } while (0)
+
+constexpr int kRingSlots = 4;
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+struct Agent {
+  int32_t len = -1;       // -1: not registered
+  bool resident = false;
+  std::vector<int32_t> pages;
+  uint64_t ready_seq = 0; // reload/offload call the next reader must wait for
+  uint64_t last_use = 0;  // last call that read or wrote the pages
+};
+
+struct Request {
+  bool open = false;
+  int32_t agent = -1;
+  int32_t len = 0;
+  std::vector<int32_t> pages;
+  uint64_t last_use = 0;
+};
+
+struct Slot {
+  uint8_t* host = nullptr;   // pinned staging
+  uint8_t* dev = nullptr;    // device copy (workspace)
+  cudaEvent_t done = nullptr;
+  uint64_t seq = 0;          // call that used the slot last (0: never)
+};
+
+// Sizes of one plan: number of records per section.
+struct PlanSizes {
+  int64_t pages = 0, append = 0, dense_tok = 0, dense = 0, suffix = 0, merge = 0;
+};
+
+struct PlanLayout {
+  size_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, total;
+};
+
+PlanLayout layout_of(const PlanSizes& s) {
+  PlanLayout l;
+  size_t o = align_up(sizeof(PlanHeader), 64);
+  l.off_pages = o;
+  o = align_up(o + s.pages * 4, 64);
+  l.off_append = o;
+  o = align_up(o + s.append * sizeof(AppendRow), 64);
+  l.off_dense_tok = o;
+  o = align_up(o + s.dense_tok * sizeof(DenseTok), 64);
+  l.off_dense = o;
+  o = align_up(o + s.dense * sizeof(DenseItem), 64);
+  l.off_suffix = o;
+  o = align_up(o + s.suffix * sizeof(SuffixItem), 64);
+  l.off_merge = o;
+  o = align_up(o + s.merge * sizeof(MergeTok), 64);
+  l.total = o;
+  return l;
+}
+
+}  // namespace
+
+struct tpa_ctx {
+  tpa_config cfg{};
+  int hq = 0, hkv = 0, d = 0, group = 0;
+  bool plan_only = false;
+  int64_t max_pages_per_seq = 0;
+  int max_splits = 32;
+
+  std::vector<int32_t> free_pages;   // used as a queue: next page at free_head
+  size_t free_head = 0;
+  std::vector<uint64_t> page_tag;    // call seq that may still read the page
+  std::vector<Agent> agents;
+  std::vector<Request> reqs;
+
+  // device side
+  int device = 0;
+  int num_sms = 148;
+  CUtensorMap tmap_k{}, tmap_v{};
+  PoolGeom pool{};
+  cudaStream_t fork_stream = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  uint32_t* status = nullptr;
+  float* part_o = nullptr;
+  float* part_lse = nullptr;
+  int64_t part_slots = 0;
+  size_t plan_cap = 0;
+  Slot ring[kRingSlots];
+  int ring_pos = 0;
+  uint64_t seq = 0;
+  uint64_t chain_seq = 0;            // last chain (ordered) call
+  cudaStream_t chain_stream = nullptr;
+
+  // options and statistics
+  int decode_mode = 0;
+  int prefix_splits = 0;
+  int suffix_split_keys = 0;
+  int concurrent = 1;
+  int64_t last_dense = 0, last_suffix = 0, last_launches = 0;
+
+  // scratch for planning (reused to avoid allocations)
+  std::vector<uint8_t> scratch;
+};
+
+namespace {
+
+// ------------------------------------------------------------------ helpers
+
+bool valid_shape(const tpa_config* c) {
+  if (!c) return false;
+  if (c->page_size != kPage) return false;
+  if (c->head_dim != 64 && c->head_dim != 128) return false;
+  if (c->num_kv_heads <= 0 || c->num_q_heads <= 0) return false;
+  if (c->num_q_heads % c->num_kv_heads) return false;
+  const int g = c->num_q_heads / c->num_kv_heads;
+  if (g != 4 && g != 8) return false;
+  return true;
+}
+
+int64_t max_pages_of(const tpa_config* c) { return cdiv(c->max_seq_len + 1, kPage) + 1; }
+
+int splits_of(const tpa_config* c) { return c->max_splits > 0 ? c->max_splits : 32; }
+
+PlanSizes plan_capacity(const tpa_config* c) {
+  const int64_t g = c->num_q_heads / c->num_kv_heads;
+  const int64_t tpt = kTileRows / g;
+  const int64_t T = c->max_tokens;
+  const int64_t A = std::min<int64_t>(c->max_agents, T);
+  const int64_t S = splits_of(c);
+  PlanSizes s;
+  s.pages = (T + A) * max_pages_of(c);
+  s.append = T;
+  s.dense_tok = T;
+  s.dense = c->num_kv_heads * ((cdiv(T, tpt) + A) * S + T + cdiv(T, tpt));
+  s.suffix = T * c->num_kv_heads * S;
+  s.merge = T;
+  return s;
+}
+
+// Wait on the device (stream `s`) for call `seq` if it may still be running.
+void wait_for_seq(tpa_ctx* ctx, uint64_t seq, cudaStream_t s) {
+  if (seq == 0 || ctx->plan_only) return;
+  for (auto& sl : ctx->ring) {
+    if (sl.seq == seq) {
+      if (cudaEventQuery(sl.done) == cudaErrorNotReady) cudaStreamWaitEvent(s, sl.done, 0);
+      else (void)cudaGetLastError();
+      return;
+    }
+  }
+  // not in the ring any more: its slot was recycled after a host-side wait
+}
+
+// Take `n` pages from the free list; returns the highest reuse tag.
+uint64_t take_pages(tpa_ctx* ctx, int64_t n, std::vector<int32_t>& out) {
+  uint64_t tag = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    const int32_t pg = ctx->free_pages[ctx->free_head++];
+    tag = std::max(tag, ctx->page_tag[pg]);
+    out.push_back(pg);
+  }
+  return tag;
+}
+
+void give_pages(tpa_ctx* ctx, std::vector<int32_t>& pages, uint64_t tag) {
+  // compact the consumed head before appending
+  if (ctx->free_head > 0 && ctx->free_head * 2 > ctx->free_pages.size()) {
+    ctx->free_pages.erase(ctx->free_pages.begin(), ctx->free_pages.begin() + ctx->free_head);
+    ctx->free_head = 0;
+  }
+  for (int32_t pg : pages) {
+    ctx->page_tag[pg] = std::max(ctx->page_tag[pg], tag);
+    ctx->free_pages.push_back(pg);
+  }
+  pages.clear();
+}
+
+int64_t free_count(const tpa_ctx* ctx) {
+  return static_cast<int64_t>(ctx->free_pages.size() - ctx->free_head);
+}
+
+// Acquire the next plan slot (host-blocking only if kRingSlots calls are in flight).
+Slot* acquire_slot(tpa_ctx* ctx) {
+  Slot* s = &ctx->ring[ctx->ring_pos];
+  ctx->ring_pos = (ctx->ring_pos + 1) % kRingSlots;
+  if (!ctx->plan_only && s->seq != 0) cudaEventSynchronize(s->done);
+  return s;
+}
+
+// Plan blob writer over a slot's host buffer.
+struct PlanWriter {
+  uint8_t* base;
+  PlanLayout lay;
+  PlanHeader* hdr;
+  int32_t* pages;
+  AppendRow* append;
+  DenseTok* dtok;
+  DenseItem* dense;
+  SuffixItem* suffix;
+  MergeTok* merge;
+  PlanWriter(uint8_t* b, const PlanLayout& l) : base(b), lay(l) {
+    hdr = reinterpret_cast<PlanHeader*>(b);
+    std::memset(hdr, 0, sizeof(PlanHeader));
+    pages = reinterpret_cast<int32_t*>(b + l.off_pages);
+    append = reinterpret_cast<AppendRow*>(b + l.off_append);
+    dtok = reinterpret_cast<DenseTok*>(b + l.off_dense_tok);
+    dense = reinterpret_cast<DenseItem*>(b + l.off_dense);
+    suffix = reinterpret_cast<SuffixItem*>(b + l.off_suffix);
+    merge = reinterpret_cast<MergeTok*>(b + l.off_merge);
+  }
+};
+
+template <class T>
+const T* dev_ptr(const Slot* s, size_t off) {
+  return reinterpret_cast<const T*>(s->dev + off);
+}
+
+int check_batch(tpa_ctx* ctx, int32_t n, const int32_t* reqs, bool need_resident) {
+  if (n <= 0 || !reqs) return fail(TPA_ERR_INVALID_ARG, "empty batch");
+  if (n > ctx->cfg.max_tokens) return fail(TPA_ERR_CAPACITY, "batch of %d > max_tokens", n);
+  for (int i = 0; i < n; ++i) {
+    const int32_t r = reqs[i];
+    if (r < 0 || r >= ctx->cfg.max_requests) return fail(TPA_ERR_INVALID_ARG, "request id %d", r);
+    if (!ctx->reqs[r].open) return fail(TPA_ERR_STATE, "request %d is not open", r);
+    if (need_resident && !ctx->agents[ctx->reqs[r].agent].resident)
+      return fail(TPA_ERR_NOT_RESIDENT, "prefix of agent %d (request %d) is not resident",
+                  ctx->reqs[r].agent, r);
+  }
+  std::vector<int32_t> sorted(reqs, reqs + n);
+  std::sort(sorted.begin(), sorted.end());
+  for (int i = 1; i < n; ++i)
+    if (sorted[i] == sorted[i - 1]) return fail(TPA_ERR_INVALID_ARG, "request %d twice", sorted[i]);
+  return TPA_OK;
+}
+
+// Begin a chain call on `s`: order after the previous chain call.
+void chain_begin(tpa_ctx* ctx, cudaStream_t s) {
+  if (ctx->plan_only) return;
+  if (ctx->chain_seq && ctx->chain_stream != s) wait_for_seq(ctx, ctx->chain_seq, s);
+}
+
+int upload(tpa_ctx* ctx, Slot* sl, size_t bytes, cudaStream_t s) {
+  if (ctx->plan_only) return TPA_OK;
+  CUDA_TRY(cudaMemcpyAsync(sl->dev, sl->host, bytes, cudaMemcpyHostToDevice, s));
+  return TPA_OK;
+}
+
+int finish_call(tpa_ctx* ctx, Slot* sl, cudaStream_t s, bool chain) {
+  sl->seq = ctx->seq;
+  if (chain) {
+    ctx->chain_seq = ctx->seq;
+    ctx->chain_stream = s;
+  }
+  if (ctx->plan_only) return TPA_OK;
+  CUDA_TRY(cudaEventRecord(sl->done, s));
+  return TPA_OK;
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+
+extern "C" {
+
+const char* tpa_last_error(void) { return g_err.c_str(); }
+
+size_t tpa_workspace_size(const tpa_config* cfg) {
+  if (!valid_shape(cfg) || cfg->max_tokens <= 0 || cfg->max_seq_len <= 0) return 0;
+  const PlanLayout lay = layout_of(plan_capacity(cfg));
+  const int64_t slots = static_cast<int64_t>(cfg->max_tokens) * cfg->num_q_heads * splits_of(cfg);
+  size_t total = kAlign;                                     // status word
+  total += kRingSlots * align_up(lay.total, kAlign);         // plan ring
+  total += align_up(slots * cfg->head_dim * sizeof(float), kAlign);
+  total += align_up(slots * sizeof(float), kAlign);
+  return total;
+}
+
+int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
+  if (!cfg || !out) return fail(TPA_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  if (!valid_shape(cfg))
+    return fail(TPA_ERR_UNSUPPORTED, "supported: page 16, head_dim 64/128, group 4/8");
+  if (cfg->num_pages <= 0 || cfg->max_agents <= 0 || cfg->max_requests <= 0 ||
+      cfg->max_tokens <= 0 || cfg->max_seq_len <= 0 || cfg->max_splits < 0)
+    return fail(TPA_ERR_INVALID_ARG, "sizes must be positive");
+  if (cfg->num_pages * cfg->num_kv_heads >= (1ll << 31))
+    return fail(TPA_ERR_UNSUPPORTED, "num_pages * num_kv_heads must be < 2^31");
+  const bool plan_only = (cfg->flags & TPA_FLAG_PLAN_ONLY) != 0;
+  if (!plan_only) {
+    if (!cfg->k_pool || !cfg->v_pool || !cfg->workspace)
+      return fail(TPA_ERR_INVALID_ARG, "pools and workspace are required");
+    if ((reinterpret_cast<uintptr_t>(cfg->k_pool) | reinterpret_cast<uintptr_t>(cfg->v_pool)) & 15)
+      return fail(TPA_ERR_INVALID_ARG, "pools must be 16-byte aligned");
+    if (reinterpret_cast<uintptr_t>(cfg->workspace) & (kAlign - 1))
+      return fail(TPA_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    if (cfg->workspace_bytes < tpa_workspace_size(cfg))
+      return fail(TPA_ERR_INVALID_ARG, "workspace of %zu bytes < %zu needed", cfg->workspace_bytes,
+                  tpa_workspace_size(cfg));
+  }
+
+  tpa_ctx* ctx = new tpa_ctx();
+  ctx->cfg = *cfg;
+  ctx->hq = cfg->num_q_heads;
+  ctx->hkv = cfg->num_kv_heads;
+  ctx->d = cfg->head_dim;
+  ctx->group = ctx->hq / ctx->hkv;
+  ctx->plan_only = plan_only;
+  ctx->max_pages_per_seq = max_pages_of(cfg);
+  ctx->max_splits = splits_of(cfg);
+  ctx->agents.resize(cfg->max_agents);
+  ctx->reqs.resize(cfg->max_requests);
+  ctx->page_tag.assign(cfg->num_pages, 0);
+  ctx->free_pages.resize(cfg->num_pages);
+  for (int64_t i = 0; i < cfg->num_pages; ++i) ctx->free_pages[i] = static_cast<int32_t>(i);
+  if (cfg->page_order_seed) {
+    // seeded Fisher-Yates with splitmix64: a fragmented pool, same on every host
+    uint64_t x = cfg->page_order_seed;
+    auto next = [&x]() {
+      uint64_t z = (x += 0x9E3779B97F4A7C15ull);
+      z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+      z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+      return z ^ (z >> 31);
+    };
+    for (int64_t i = cfg->num_pages - 1; i > 0; --i) {
+      const int64_t j = static_cast<int64_t>(next() % static_cast<uint64_t>(i + 1));
+      std::swap(ctx->free_pages[i], ctx->free_pages[j]);
+    }
+  }
+
+  const PlanLayout lay = layout_of(plan_capacity(cfg));
+  ctx->plan_cap = align_up(lay.total, kAlign);
+  ctx->part_slots = static_cast<int64_t>(cfg->max_tokens) * ctx->hq * ctx->max_splits;
+
+  if (plan_only) {
+    for (auto& s : ctx->ring) s.host = static_cast<uint8_t*>(std::malloc(ctx->plan_cap));
+    *out = ctx;
+    return TPA_OK;
+  }
+
+  auto cleanup = [ctx](int code) {
+    tpa_destroy(ctx);
+    return code;
+  };
+  int rc;
+  cudaError_t e;
+  if ((e = cudaGetDevice(&ctx->device)) != cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e)));
+  if ((e = cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, ctx->device)) !=
+      cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "SM count: %s", cudaGetErrorString(e)));
+  if ((e = tpa::init_kernels()) != cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "kernel attributes: %s", cudaGetErrorString(e)));
+
+  // TMA descriptors: 3-D view (d, 16 slots, pages*hkv) of each pool, 64x16 boxes
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if ((e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                            &q)) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess || !fn)
+    return cleanup(fail(TPA_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable"));
+  auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  const cuuint64_t dims[3] = {static_cast<cuuint64_t>(ctx->d), static_cast<cuuint64_t>(kPage),
+                              static_cast<cuuint64_t>(cfg->num_pages * ctx->hkv)};
+  const cuuint64_t strides[2] = {static_cast<cuuint64_t>(ctx->d) * 2,
+                                 static_cast<cuuint64_t>(kPage) * ctx->d * 2};
+  const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(kPage), 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  for (int w = 0; w < 2; ++w) {
+    CUresult r = encode(w ? &ctx->tmap_v : &ctx->tmap_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                        w ? cfg->v_pool : cfg->k_pool, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cleanup(fail(TPA_ERR_CUDA, "cuTensorMapEncodeTiled: %d", (int)r));
+  }
+  ctx->pool = PoolGeom{cfg->k_pool, cfg->v_pool, cfg->num_pages, ctx->hkv, ctx->d};
+
+  // workspace carve-up
+  uint8_t* ws = static_cast<uint8_t*>(cfg->workspace);
+  ctx->status = reinterpret_cast<uint32_t*>(ws);
+  size_t off = kAlign;
+  for (auto& s : ctx->ring) {
+    s.dev = ws + off;
+    off += ctx->plan_cap;
+  }
+  ctx->part_o = reinterpret_cast<float*>(ws + off);
+  off += align_up(ctx->part_slots * ctx->d * sizeof(float), kAlign);
+  ctx->part_lse = reinterpret_cast<float*>(ws + off);
+
+  for (auto& s : ctx->ring) {
+    if ((e = cudaHostAlloc(reinterpret_cast<void**>(&s.host), ctx->plan_cap, cudaHostAllocDefault)) !=
+        cudaSuccess)
+      return cleanup(fail(TPA_ERR_CUDA, "pinned staging: %s", cudaGetErrorString(e)));
+    if ((e = cudaEventCreateWithFlags(&s.done, cudaEventDisableTiming)) != cudaSuccess)
+      return cleanup(fail(TPA_ERR_CUDA, "event: %s", cudaGetErrorString(e)));
+  }
+  if ((e = cudaStreamCreateWithFlags(&ctx->fork_stream, cudaStreamNonBlocking)) != cudaSuccess ||
+      (e = cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming)) != cudaSuccess ||
+      (e = cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming)) != cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "streams: %s", cudaGetErrorString(e)));
+  if ((e = cudaMemsetAsync(ctx->status, 0, sizeof(uint32_t), 0)) != cudaSuccess ||
+      (e = cudaStreamSynchronize(0)) != cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "status init: %s", cudaGetErrorString(e)));
+  (void)rc;
+  *out = ctx;
+  return TPA_OK;
+}
+
+int tpa_destroy(tpa_ctx* ctx) {
+  if (!ctx) return TPA_OK;
+  if (ctx->plan_only) {
+    for (auto& s : ctx->ring) std::free(s.host);
+  } else {
+    for (auto& s : ctx->ring) {
+      if (s.done) {
+        if (s.seq) cudaEventSynchronize(s.done);
+        cudaEventDestroy(s.done);
+      }
+      if (s.host) cudaFreeHost(s.host);
+    }
+    if (ctx->fork_stream) {
+      cudaStreamSynchronize(ctx->fork_stream);
+      cudaStreamDestroy(ctx->fork_stream);
+    }
+    if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
+    if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
+  }
+  delete ctx;
+  return TPA_OK;
+}
+
+// ---------------------------------------------------------------- prefixes
+
+int tpa_prefix_register(tpa_ctx* ctx, int32_t agent, int32_t len) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  if (agent < 0 || agent >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", agent);
+  if (len < 0 || len > ctx->cfg.max_seq_len) return fail(TPA_ERR_INVALID_ARG, "prefix length %d", len);
+  Agent& a = ctx->agents[agent];
+  if (a.len >= 0) return fail(TPA_ERR_STATE, "agent %d is already registered", agent);
+  const int64_t need = cdiv(len, kPage);
+  if (need > free_count(ctx))
+    return fail(TPA_ERR_NO_SPACE, "prefix needs %lld pages, %lld free", (long long)need,
+                (long long)free_count(ctx));
+  a.pages.clear();
+  const uint64_t tag = take_pages(ctx, need, a.pages);
+  a.len = len;
+  a.resident = true;
+  a.ready_seq = 0;
+  a.last_use = tag;  // a later writer must wait for the pages' previous readers
+  return TPA_OK;
+}
+
+static int page_copy_call(tpa_ctx* ctx, const std::vector<int32_t>& pages, int len, int to_pages,
+                          const void* k_in, const void* v_in, void* k_out, void* v_out,
+                          cudaStream_t s, bool chain, uint64_t wait_seq, Slot** used) {
+  Slot* sl = acquire_slot(ctx);
+  ++ctx->seq;
+  PlanSizes sz;
+  sz.pages = static_cast<int64_t>(pages.size());
+  const PlanLayout lay = layout_of(sz);
+  if (lay.total > ctx->plan_cap) return fail(TPA_ERR_CAPACITY, "page list too long");
+  PlanWriter w(sl->host, lay);
+  w.hdr->n_pages = static_cast<int32_t>(pages.size());
+  std::memcpy(w.pages, pages.data(), pages.size() * 4);
+  if (chain) chain_begin(ctx, s);
+  wait_for_seq(ctx, wait_seq, s);
+  int rc = upload(ctx, sl, lay.total, s);
+  if (rc) return rc;
+  if (!ctx->plan_only) {
+    CUDA_TRY(launch_page_copy(dev_ptr<int32_t>(sl, lay.off_pages), len, to_pages, k_in, v_in, k_out,
+                              v_out, ctx->pool, ctx->status, s));
+  }
+  ctx->last_launches = 1;
+  if (used) *used = sl;
+  return finish_call(ctx, sl, s, chain);
+}
+
+static int resolve_host_ptr(const void* p, const void** dev) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return fail(TPA_ERR_INVALID_ARG, "host pointer %p is not known to CUDA", p);
+  }
+  if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) {
+    *dev = p;
+    return TPA_OK;
+  }
+  if (at.type != cudaMemoryTypeHost)
+    return fail(TPA_ERR_INVALID_ARG, "host memory %p is not pinned", p);
+  void* d = nullptr;
+  if (cudaHostGetDevicePointer(&d, const_cast<void*>(p), 0) != cudaSuccess || !d) {
+    (void)cudaGetLastError();
+    return fail(TPA_ERR_INVALID_ARG, "pinned host memory %p is not mapped", p);
+  }
+  *dev = d;
+  return TPA_OK;
+}
+
+int tpa_prefix_write(tpa_ctx* ctx, int32_t agent, const void* k, const void* v, void* stream) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  if (agent < 0 || agent >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", agent);
+  Agent& a = ctx->agents[agent];
+  if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
+  if (!a.resident) return fail(TPA_ERR_NOT_RESIDENT, "agent %d is not resident", agent);
+  if (a.len == 0) return TPA_OK;
+  if (!k || !v) return fail(TPA_ERR_INVALID_ARG, "null source");
+  const void* kd = k;
+  const void* vd = v;
+  if (!ctx->plan_only) {
+    int rc;
+    if ((rc = resolve_host_ptr(k, &kd)) || (rc = resolve_host_ptr(v, &vd))) return rc;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  wait_for_seq(ctx, a.ready_seq, s);
+  const int rc = page_copy_call(ctx, a.pages, a.len, 1, kd, vd, nullptr, nullptr, s, true,
+                                a.last_use, nullptr);
+  if (rc) return rc;
+  a.last_use = ctx->seq;
+  a.ready_seq = 0;
+  return TPA_OK;
+}
+
+int tpa_prefix_evict(tpa_ctx* ctx, int32_t agent) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  if (agent < 0 || agent >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", agent);
+  Agent& a = ctx->agents[agent];
+  if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
+  if (!a.resident) return fail(TPA_ERR_NOT_RESIDENT, "agent %d is already evicted", agent);
+  give_pages(ctx, a.pages, std::max(a.last_use, a.ready_seq));
+  a.resident = false;
+  return TPA_OK;
+}
+
+int tpa_prefix_reload(tpa_ctx* ctx, int32_t agent, const void* host_k, const void* host_v,
+                      void* side_stream, void* done_event) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  if (agent < 0 || agent >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", agent);
+  Agent& a = ctx->agents[agent];
+  if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
+  if (a.resident) return fail(TPA_ERR_STATE, "agent %d is already resident", agent);
+  if (a.len > 0 && (!host_k || !host_v)) return fail(TPA_ERR_INVALID_ARG, "null source");
+  const void* kd = host_k;
+  const void* vd = host_v;
+  if (!ctx->plan_only && a.len > 0) {
+    int rc;
+    if ((rc = resolve_host_ptr(host_k, &kd)) || (rc = resolve_host_ptr(host_v, &vd))) return rc;
+  }
+  const int64_t need = cdiv(a.len, kPage);
+  if (need > free_count(ctx))
+    return fail(TPA_ERR_NO_SPACE, "reload needs %lld pages, %lld free", (long long)need,
+                (long long)free_count(ctx));
+  std::vector<int32_t> pages;
+  const uint64_t tag = take_pages(ctx, need, pages);
+  cudaStream_t s = static_cast<cudaStream_t>(side_stream);
+  const int rc = page_copy_call(ctx, pages, a.len, 1, kd, vd, nullptr, nullptr, s, false,
+                                std::max(tag, a.last_use), nullptr);
+  if (rc) {
+    // give the pages back untouched (nothing was queued that writes them)
+    for (auto it = pages.rbegin(); it != pages.rend(); ++it) ctx->free_pages[--ctx->free_head] = *it;
+    return rc;
+  }
+  a.pages = std::move(pages);
+  a.resident = true;
+  a.ready_seq = ctx->seq;
+  a.last_use = ctx->seq;
+  if (done_event && !ctx->plan_only) CUDA_TRY(cudaEventRecord(static_cast<cudaEvent_t>(done_event), s));
+  return TPA_OK;
+}
+
+int tpa_prefix_offload(tpa_ctx* ctx, int32_t agent, void* host_k, void* host_v, void* side_stream,
+                       void* done_event) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  if (agent < 0 || agent >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", agent);
+  Agent& a = ctx->agents[agent];
+  if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
+  if (!a.resident) return fail(TPA_ERR_NOT_RESIDENT, "agent %d is not resident", agent);
+  if (a.len > 0 && (!host_k || !host_v)) return fail(TPA_ERR_INVALID_ARG, "null destination");
+  const void* kd = host_k;
+  const void* vd = host_v;
+  if (!ctx->plan_only && a.len > 0) {
+    int rc;
+    if ((rc = resolve_host_ptr(host_k, &kd)) || (rc = resolve_host_ptr(host_v, &vd))) return rc;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(side_stream);
+  // the pages' last writer/readers must finish before the copy reads them
+  wait_for_seq(ctx, ctx->chain_seq, s);
+  const int rc = page_copy_call(ctx, a.pages, a.len, 0, nullptr, nullptr, const_cast<void*>(kd),
+                                const_cast<void*>(vd), s, false, std::max(a.ready_seq, a.last_use),
+                                nullptr);
+  if (rc) return rc;
+  a.last_use = ctx->seq;
+  give_pages(ctx, a.pages, ctx->seq);
+  a.resident = false;
+  a.ready_seq = 0;
+  if (done_event && !ctx->plan_only) CUDA_TRY(cudaEventRecord(static_cast<cudaEvent_t>(done_event), s));
+  return TPA_OK;
+}
+
+// ---------------------------------------------------------------- requests
+
+int tpa_request_open(tpa_ctx* ctx, int32_t req, int32_t agent) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  if (req < 0 || req >= ctx->cfg.max_requests) return fail(TPA_ERR_INVALID_ARG, "request id %d", req);
+  if (agent < 0 || agent >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", agent);
+  if (ctx->reqs[req].open) return fail(TPA_ERR_STATE, "request %d is already open", req);
+  if (ctx->agents[agent].len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
+  Request& r = ctx->reqs[req];
+  r = Request();
+  r.open = true;
+  r.agent = agent;
+  return TPA_OK;
+}
+
+int tpa_request_close(tpa_ctx* ctx, int32_t req) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  if (req < 0 || req >= ctx->cfg.max_requests) return fail(TPA_ERR_INVALID_ARG, "request id %d", req);
+  Request& r = ctx->reqs[req];
+  if (!r.open) return fail(TPA_ERR_STATE, "request %d is not open", req);
+  give_pages(ctx, r.pages, r.last_use);
+  r = Request();
+  return TPA_OK;
+}
+
+// Reserve pages for appending ntok[i] tokens to request reqs[i]; all or nothing.
+static int reserve_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* ntok,
+                          uint64_t* tag) {
+  int64_t need = 0;
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    if (ntok[i] < 0) return fail(TPA_ERR_INVALID_ARG, "negative token count");
+    if (static_cast<int64_t>(r.len) + ntok[i] > ctx->cfg.max_seq_len)
+      return fail(TPA_ERR_CAPACITY, "suffix of request %d would exceed max_seq_len", reqs[i]);
+    need += cdiv(r.len + ntok[i], kPage) - static_cast<int64_t>(r.pages.size());
+  }
+  if (need > free_count(ctx))
+    return fail(TPA_ERR_NO_SPACE, "append needs %lld pages, %lld free", (long long)need,
+                (long long)free_count(ctx));
+  uint64_t t = 0;
+  for (int i = 0; i < n; ++i) {
+    Request& r = ctx->reqs[reqs[i]];
+    const int64_t add = cdiv(r.len + ntok[i], kPage) - static_cast<int64_t>(r.pages.size());
+    t = std::max(t, take_pages(ctx, add, r.pages));
+  }
+  *tag = t;
+  return TPA_OK;
+}
+
+static void write_append_rows(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* ntok,
+                              AppendRow* rows) {
+  int64_t row = 0;
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    for (int t = 0; t < ntok[i]; ++t, ++row) {
+      const int pos = r.len + t;
+      rows[row] = AppendRow{static_cast<int32_t>(row), r.pages[pos / kPage], pos % kPage, 0};
+    }
+  }
+}
+
+int tpa_kv_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* ntok,
+                  const void* k_new, const void* v_new, void* stream) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  int rc = check_batch(ctx, n, reqs, false);
+  if (rc) return rc;
+  if (!ntok) return fail(TPA_ERR_INVALID_ARG, "null token counts");
+  int64_t total = 0;
+  for (int i = 0; i < n; ++i) total += ntok[i] > 0 ? ntok[i] : 0;
+  if (total > ctx->cfg.max_tokens) return fail(TPA_ERR_CAPACITY, "%lld tokens > max_tokens", (long long)total);
+  if (total > 0 && (!k_new || !v_new)) return fail(TPA_ERR_INVALID_ARG, "null K/V");
+  uint64_t tag = 0;
+  if ((rc = reserve_append(ctx, n, reqs, ntok, &tag))) return rc;
+  Slot* sl = acquire_slot(ctx);
+  ++ctx->seq;
+  PlanSizes sz;
+  sz.append = total;
+  const PlanLayout lay = layout_of(sz);
+  PlanWriter w(sl->host, lay);
+  w.hdr->n_append = static_cast<int32_t>(total);
+  write_append_rows(ctx, n, reqs, ntok, w.append);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  chain_begin(ctx, s);
+  wait_for_seq(ctx, tag, s);
+  if ((rc = upload(ctx, sl, lay.total, s))) return rc;
+  if (!ctx->plan_only)
+    CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
+                           v_new, ctx->pool, ctx->status, s));
+  for (int i = 0; i < n; ++i) {
+    Request& r = ctx->reqs[reqs[i]];
+    r.len += ntok[i];
+    r.last_use = ctx->seq;
+  }
+  ctx->last_launches = 1;
+  ctx->last_dense = ctx->last_suffix = 0;
+  return finish_call(ctx, sl, s, true);
+}
+
+// ------------------------------------------------------------- attention
+
+namespace {
+
+struct AgentGroup {
+  int32_t agent;
+  std::vector<int32_t> toks;  // positions in the batch
+  int32_t page_off = 0;       // prefix pages in the plan's page list
+  int32_t n_split = 0;        // key splits of the prefix level
+  int32_t tiles_per_split = 0;
+};
+
+}  // namespace
+
+// Build and launch a decode step (cascade or flat).
+int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, const void* k_new,
+               const void* v_new, void* out, float* lse, void* stream) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  int rc = check_batch(ctx, n, reqs, true);
+  if (rc) return rc;
+  if (!ctx->plan_only && (!q || !k_new || !v_new || !out || !lse))
+    return fail(TPA_ERR_INVALID_ARG, "null tensor");
+  const int G = ctx->group, hkv = ctx->hkv, hq = ctx->hq;
+  const int tpt = kTileRows / G;
+  const bool flat = ctx->decode_mode == 1;
+
+  // group tokens by agent (first appearance order)
+  std::vector<AgentGroup> groups;
+  {
+    std::unordered_map<int32_t, int> gi;
+    for (int i = 0; i < n; ++i) {
+      const int32_t a = ctx->reqs[reqs[i]].agent;
+      auto it = gi.find(a);
+      if (it == gi.end()) {
+        gi[a] = static_cast<int>(groups.size());
+        groups.push_back(AgentGroup{a, {i}});
+      } else {
+        groups[it->second].toks.push_back(i);
+      }
+    }
+  }
+
+  // split sizes
+  int64_t max_len = 0, sum_keys = 0, max_prefix = 0;
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    max_len = std::max<int64_t>(max_len, r.len + 1);
+    sum_keys += r.len + 1;
+    max_prefix = std::max<int64_t>(max_prefix, ctx->agents[r.agent].len);
+    if (flat) sum_keys += ctx->agents[r.agent].len;
+  }
+  int n_units = 0;  // dense (agent, kv head, q tile) units
+  if (!flat)
+    for (auto& g : groups)
+      if (ctx->agents[g.agent].len > 0) n_units += hkv * static_cast<int>(cdiv(g.toks.size(), tpt));
+  int64_t split_keys = ctx->suffix_split_keys;
+  if (split_keys <= 0) {
+    // about two items per resident warp, 64..1024 keys each
+    const int64_t warps = static_cast<int64_t>(ctx->num_sms) * 8;
+    split_keys = cdiv(sum_keys * hkv, 2 * warps);
+    split_keys = std::min<int64_t>(std::max<int64_t>(split_keys, 64), 1024);
+  }
+  split_keys = cdiv(split_keys, kPage) * kPage;
+  for (auto& g : groups) {
+    const int64_t lp = ctx->agents[g.agent].len;
+    if (flat || lp == 0) continue;
+    const int64_t tiles = cdiv(lp, kTileKeys);
+    int64_t ns = ctx->prefix_splits;
+    if (ns <= 0) ns = std::max<int64_t>(1, cdiv(ctx->num_sms, std::max(1, n_units)));
+    ns = std::min<int64_t>(ns, tiles);
+    g.tiles_per_split = static_cast<int32_t>(cdiv(tiles, ns));
+    g.n_split = static_cast<int32_t>(cdiv(tiles, g.tiles_per_split));
+  }
+  // keep every token's partial count within max_splits
+  {
+    int64_t worst = 0;
+    for (int i = 0; i < n; ++i) {
+      const Request& r = ctx->reqs[reqs[i]];
+      const int64_t lp = ctx->agents[r.agent].len;
+      int64_t nsp = 0;
+      for (auto& g : groups)
+        if (g.agent == r.agent) nsp = g.n_split;
+      const int64_t keys_flat = flat ? lp : 0;
+      worst = std::max(worst, nsp + cdiv(r.len + 1, split_keys) + cdiv(keys_flat, split_keys));
+      if (nsp >= ctx->max_splits) return fail(TPA_ERR_CAPACITY, "prefix splits exceed max_splits");
+    }
+    while (worst > ctx->max_splits) {
+      split_keys *= 2;
+      worst = 0;
+      for (int i = 0; i < n; ++i) {
+        const Request& r = ctx->reqs[reqs[i]];
+        const int64_t lp = ctx->agents[r.agent].len;
+        int64_t nsp = 0;
+        for (auto& g : groups)
+          if (g.agent == r.agent) nsp = g.n_split;
+        worst = std::max(worst, nsp + cdiv(r.len + 1, split_keys) + cdiv(flat ? lp : 0, split_keys));
+      }
+    }
+  }
+
+  std::vector<int32_t> ones(n, 1);
+
+  // sizes (suffix page counts after this step's append)
+  PlanSizes sz;
+  sz.append = n;
+  sz.merge = n;
+  sz.dense_tok = n;
+  for (auto& g : groups) sz.pages += ctx->agents[g.agent].pages.size();
+  for (int i = 0; i < n; ++i) sz.pages += cdiv(ctx->reqs[reqs[i]].len + 1, kPage);
+  int64_t n_dense = 0, n_suffix = 0;
+  for (auto& g : groups) n_dense += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) * g.n_split;
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    n_suffix += hkv * (cdiv(r.len + 1, split_keys) + (flat ? cdiv(ctx->agents[r.agent].len, split_keys) : 0));
+  }
+  sz.dense = n_dense;
+  sz.suffix = n_suffix;
+  const PlanLayout lay = layout_of(sz);
+  if (lay.total > ctx->plan_cap) return fail(TPA_ERR_CAPACITY, "plan of %zu bytes > %zu", lay.total, ctx->plan_cap);
+
+  // partial slots per token
+  std::vector<int32_t> nsp_of(n, 0), slot_base(n), n_slots(n);
+  for (auto& g : groups)
+    for (int32_t i : g.toks) nsp_of[i] = g.n_split;
+  int64_t slots = 0;
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    const int64_t lp = ctx->agents[r.agent].len;
+    n_slots[i] = static_cast<int32_t>(nsp_of[i] + cdiv(r.len + 1, split_keys) + (flat ? cdiv(lp, split_keys) : 0));
+    slot_base[i] = static_cast<int32_t>(slots);
+    slots += static_cast<int64_t>(hq) * n_slots[i];
+  }
+  if (slots > ctx->part_slots) return fail(TPA_ERR_CAPACITY, "partial slots exhausted");
+
+  // pages for the new tokens (all checks are done: from here on only CUDA errors can fail)
+  uint64_t tag = 0;
+  if ((rc = reserve_append(ctx, n, reqs, ones.data(), &tag))) return rc;
+
+  Slot* sl = acquire_slot(ctx);
+  ++ctx->seq;
+  PlanWriter w(sl->host, lay);
+  for (int i = 0; i < n; ++i) w.merge[i] = MergeTok{i, slot_base[i], n_slots[i], 0};
+
+  // page list: prefixes, then each token's suffix (after the append)
+  int32_t np = 0;
+  for (auto& g : groups) {
+    const Agent& a = ctx->agents[g.agent];
+    g.page_off = np;
+    std::memcpy(w.pages + np, a.pages.data(), a.pages.size() * 4);
+    np += static_cast<int32_t>(a.pages.size());
+  }
+  std::vector<int32_t> suf_off(n);
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    suf_off[i] = np;
+    std::memcpy(w.pages + np, r.pages.data(), r.pages.size() * 4);
+    np += static_cast<int32_t>(r.pages.size());
+  }
+  write_append_rows(ctx, n, reqs, ones.data(), w.append);
+
+  // level 1: stacked prefix tiles
+  int32_t nt = 0, nd = 0;
+  for (auto& g : groups) {
+    if (g.n_split == 0) continue;
+    const int64_t lp = ctx->agents[g.agent].len;
+    const int nqt = static_cast<int>(cdiv(g.toks.size(), tpt));
+    for (int qt = 0; qt < nqt; ++qt) {
+      const int t0 = qt * tpt;
+      const int t1 = std::min<int>(static_cast<int>(g.toks.size()), t0 + tpt);
+      const int32_t tok_base = nt;
+      for (int t = t0; t < t1; ++t) {
+        const int i = g.toks[t];
+        w.dtok[nt++] = DenseTok{i, 0x7fffffff, slot_base[i], n_slots[i]};
+      }
+      for (int h = 0; h < hkv; ++h)
+        for (int sp = 0; sp < g.n_split; ++sp) {
+          DenseItem it{};
+          it.tok_base = tok_base;
+          it.n_tok = t1 - t0;
+          it.kv_head = h;
+          it.split = sp;
+          it.out_mode = 0;
+          it.seg_pages[0] = g.page_off;
+          it.seg_k0[0] = static_cast<int32_t>(static_cast<int64_t>(sp) * g.tiles_per_split * kTileKeys);
+          it.seg_k1[0] = static_cast<int32_t>(std::min<int64_t>(lp, static_cast<int64_t>(sp + 1) * g.tiles_per_split * kTileKeys));
+          it.seg_pages[1] = 0;
+          it.seg_k0[1] = it.seg_k1[1] = 0;
+          it.n_tiles = static_cast<int32_t>(cdiv(it.seg_k1[0] - it.seg_k0[0], kTileKeys));
+          w.dense[nd++] = it;
+        }
+    }
+  }
+  // level 2: split-KV over suffixes (and prefixes in flat mode)
+  int32_t ns = 0;
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    const int64_t keys = r.len + 1;
+    const int64_t lp = ctx->agents[r.agent].len;
+    int32_t gpo = 0;
+    for (auto& g : groups)
+      if (g.agent == r.agent) gpo = g.page_off;
+    int split = nsp_of[i];
+    for (int pass = 0; pass < 2; ++pass) {
+      const bool pre = pass == 0;
+      if (pre && !flat) continue;
+      const int64_t len = pre ? lp : keys;
+      const int32_t base = pre ? gpo : suf_off[i];
+      for (int64_t k0 = 0; k0 < len; k0 += split_keys, ++split)
+        for (int h = 0; h < hkv; ++h)
+          w.suffix[ns++] = SuffixItem{i, h, static_cast<int32_t>(base + k0 / kPage),
+                                      static_cast<int32_t>(std::min<int64_t>(split_keys, len - k0)),
+                                      slot_base[i], n_slots[i], split, 0};
+    }
+  }
+  std::stable_sort(w.suffix, w.suffix + ns,
+                   [](const SuffixItem& a, const SuffixItem& b) { return a.n_keys > b.n_keys; });
+  std::stable_sort(w.dense, w.dense + nd,
+                   [](const DenseItem& a, const DenseItem& b) { return a.n_tiles > b.n_tiles; });
+
+  PlanHeader* hd = w.hdr;
+  hd->n_pages = np;
+  hd->n_append = n;
+  hd->n_dense_tok = nt;
+  hd->n_dense = nd;
+  hd->n_suffix = ns;
+  hd->n_merge = n;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  chain_begin(ctx, s);
+  wait_for_seq(ctx, tag, s);
+  for (auto& g : groups) wait_for_seq(ctx, ctx->agents[g.agent].ready_seq, s);
+  if ((rc = upload(ctx, sl, lay.total, s))) return rc;
+
+  int launches = 0;
+  if (!ctx->plan_only) {
+    CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), n, k_new, v_new, ctx->pool,
+                           ctx->status, s));
+    ++launches;
+    const float scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(ctx->d));
+    cudaStream_t ds = s;
+    const bool fork = ctx->concurrent && nd > 0 && ns > 0;
+    if (fork) {
+      CUDA_TRY(cudaEventRecord(ctx->ev_fork, s));
+      CUDA_TRY(cudaStreamWaitEvent(ctx->fork_stream, ctx->ev_fork, 0));
+      ds = ctx->fork_stream;
+    }
+    if (nd > 0) {
+      DenseParams dp{};
+      dp.tmap_k = ctx->tmap_k;
+      dp.tmap_v = ctx->tmap_v;
+      dp.q = static_cast<const __nv_bfloat16*>(q);
+      dp.out = static_cast<__nv_bfloat16*>(out);
+      dp.lse = lse;
+      dp.part_o = ctx->part_o;
+      dp.part_lse = ctx->part_lse;
+      dp.items = dev_ptr<DenseItem>(sl, lay.off_dense);
+      dp.toks = dev_ptr<DenseTok>(sl, lay.off_dense_tok);
+      dp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
+      dp.status = ctx->status;
+      dp.num_pages = ctx->cfg.num_pages;
+      dp.hq = hq;
+      dp.hkv = hkv;
+      dp.scale_log2 = scale_log2;
+      CUDA_TRY(launch_dense(dp, nd, ctx->d, G, ds));
+      ++launches;
+    }
+    if (ns > 0) {
+      SuffixParams sp{};
+      sp.tmap_k = ctx->tmap_k;
+      sp.tmap_v = ctx->tmap_v;
+      sp.q = static_cast<const __nv_bfloat16*>(q);
+      sp.part_o = ctx->part_o;
+      sp.part_lse = ctx->part_lse;
+      sp.items = dev_ptr<SuffixItem>(sl, lay.off_suffix);
+      sp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
+      sp.queue = reinterpret_cast<uint32_t*>(sl->dev + offsetof(PlanHeader, queue));
+      sp.status = ctx->status;
+      sp.num_pages = ctx->cfg.num_pages;
+      sp.n_items = ns;
+      sp.hq = hq;
+      sp.hkv = hkv;
+      sp.scale_log2 = scale_log2;
+      CUDA_TRY(launch_suffix(sp, ctx->num_sms, ctx->d, G, s));
+      ++launches;
+    }
+    if (fork) {
+      CUDA_TRY(cudaEventRecord(ctx->ev_join, ctx->fork_stream));
+      CUDA_TRY(cudaStreamWaitEvent(s, ctx->ev_join, 0));
+    }
+    CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
+                          static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, s));
+    ++launches;
+  }
+  for (int i = 0; i < n; ++i) {
+    Request& r = ctx->reqs[reqs[i]];
+    r.len += 1;
+    r.last_use = ctx->seq;
+  }
+  for (auto& g : groups) ctx->agents[g.agent].last_use = ctx->seq;
+  ctx->last_dense = nd;
+  ctx->last_suffix = ns;
+  ctx->last_launches = launches;
+  return finish_call(ctx, sl, s, true);
+}
+
+int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* chunk_len,
+                      const void* q, const void* k_new, const void* v_new, void* out, float* lse,
+                      void* stream) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  int rc = check_batch(ctx, n, reqs, true);
+  if (rc) return rc;
+  if (!chunk_len) return fail(TPA_ERR_INVALID_ARG, "null chunk lengths");
+  int64_t total = 0;
+  for (int i = 0; i < n; ++i) {
+    if (chunk_len[i] <= 0) return fail(TPA_ERR_INVALID_ARG, "chunk length %d", chunk_len[i]);
+    total += chunk_len[i];
+  }
+  if (total > ctx->cfg.max_tokens) return fail(TPA_ERR_CAPACITY, "%lld tokens > max_tokens", (long long)total);
+  if (!ctx->plan_only && (!q || !k_new || !v_new || !out || !lse))
+    return fail(TPA_ERR_INVALID_ARG, "null tensor");
+  const int G = ctx->group, hkv = ctx->hkv, hq = ctx->hq;
+  const int tpt = kTileRows / G;
+
+  std::vector<int32_t> offset(n);
+  for (int i = 0; i < n; ++i) offset[i] = ctx->reqs[reqs[i]].len;
+
+  std::vector<int32_t> agents_seen;
+  PlanSizes sz;
+  sz.append = total;
+  sz.dense_tok = total;
+  std::unordered_map<int32_t, int32_t> agent_off;
+  for (int i = 0; i < n; ++i) {
+    const int32_t a = ctx->reqs[reqs[i]].agent;
+    if (!agent_off.count(a)) {
+      agent_off[a] = 0;
+      agents_seen.push_back(a);
+      sz.pages += ctx->agents[a].pages.size();
+    }
+    sz.pages += cdiv(offset[i] + chunk_len[i], kPage);
+    sz.dense += static_cast<int64_t>(hkv) * cdiv(chunk_len[i], tpt);
+  }
+  const PlanLayout lay = layout_of(sz);
+  if (lay.total > ctx->plan_cap) return fail(TPA_ERR_CAPACITY, "plan of %zu bytes > %zu", lay.total, ctx->plan_cap);
+  uint64_t tag = 0;
+  if ((rc = reserve_append(ctx, n, reqs, chunk_len, &tag))) return rc;
+
+  Slot* sl = acquire_slot(ctx);
+  ++ctx->seq;
+  PlanWriter w(sl->host, lay);
+  int32_t np = 0;
+  for (int32_t a : agents_seen) {
+    agent_off[a] = np;
+    const Agent& ag = ctx->agents[a];
+    std::memcpy(w.pages + np, ag.pages.data(), ag.pages.size() * 4);
+    np += static_cast<int32_t>(ag.pages.size());
+  }
+  // append rows use the positions before this call
+  {
+    int64_t row = 0;
+    for (int i = 0; i < n; ++i) {
+      const Request& r = ctx->reqs[reqs[i]];
+      for (int t = 0; t < chunk_len[i]; ++t, ++row) {
+        const int pos = offset[i] + t;
+        w.append[row] = AppendRow{static_cast<int32_t>(row), r.pages[pos / kPage], pos % kPage, 0};
+      }
+    }
+  }
+  int32_t nt = 0, nd = 0;
+  int64_t row0 = 0;
+  for (int i = 0; i < n; ++i) {
+    const Request& r = ctx->reqs[reqs[i]];
+    const int64_t lp = ctx->agents[r.agent].len;
+    const int32_t suf = np;
+    std::memcpy(w.pages + np, r.pages.data(), r.pages.size() * 4);
+    np += static_cast<int32_t>(r.pages.size());
+    const int c = chunk_len[i];
+    for (int t0 = 0; t0 < c; t0 += tpt) {
+      const int t1 = std::min(c, t0 + tpt);
+      const int32_t tok_base = nt;
+      for (int t = t0; t < t1; ++t)
+        w.dtok[nt++] = DenseTok{static_cast<int32_t>(row0 + t), offset[i] + t, 0, 0};
+      for (int h = 0; h < hkv; ++h) {
+        DenseItem it{};
+        it.tok_base = tok_base;
+        it.n_tok = t1 - t0;
+        it.kv_head = h;
+        it.out_mode = 1;
+        it.seg_pages[0] = agent_off[r.agent];
+        it.seg_k0[0] = 0;
+        it.seg_k1[0] = static_cast<int32_t>(lp);
+        it.seg_pages[1] = suf;
+        it.seg_k0[1] = 0;
+        it.seg_k1[1] = offset[i] + t1;  // keys up to the tile's last position
+        it.seg_causal[1] = 1;
+        it.n_tiles = static_cast<int32_t>(cdiv(lp, kTileKeys) + cdiv(it.seg_k1[1], kTileKeys));
+        w.dense[nd++] = it;
+      }
+    }
+    row0 += c;
+  }
+  std::stable_sort(w.dense, w.dense + nd,
+                   [](const DenseItem& a, const DenseItem& b) { return a.n_tiles > b.n_tiles; });
+  PlanHeader* hd = w.hdr;
+  hd->n_pages = np;
+  hd->n_append = static_cast<int32_t>(total);
+  hd->n_dense_tok = nt;
+  hd->n_dense = nd;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  chain_begin(ctx, s);
+  wait_for_seq(ctx, tag, s);
+  for (int32_t a : agents_seen) wait_for_seq(ctx, ctx->agents[a].ready_seq, s);
+  if ((rc = upload(ctx, sl, lay.total, s))) return rc;
+  if (!ctx->plan_only) {
+    CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
+                           v_new, ctx->pool, ctx->status, s));
+    DenseParams dp{};
+    dp.tmap_k = ctx->tmap_k;
+    dp.tmap_v = ctx->tmap_v;
+    dp.q = static_cast<const __nv_bfloat16*>(q);
+    dp.out = static_cast<__nv_bfloat16*>(out);
+    dp.lse = lse;
+    dp.part_o = ctx->part_o;
+    dp.part_lse = ctx->part_lse;
+    dp.items = dev_ptr<DenseItem>(sl, lay.off_dense);
+    dp.toks = dev_ptr<DenseTok>(sl, lay.off_dense_tok);
+    dp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
+    dp.status = ctx->status;
+    dp.num_pages = ctx->cfg.num_pages;
+    dp.hq = hq;
+    dp.hkv = hkv;
+    dp.scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(ctx->d));
+    CUDA_TRY(launch_dense(dp, nd, ctx->d, G, s));
+  }
+  for (int i = 0; i < n; ++i) {
+    Request& r = ctx->reqs[reqs[i]];
+    r.len += chunk_len[i];
+    r.last_use = ctx->seq;
+  }
+  for (int32_t a : agents_seen) ctx->agents[a].last_use = ctx->seq;
+  ctx->last_dense = nd;
+  ctx->last_suffix = 0;
+  ctx->last_launches = 2;
+  return finish_call(ctx, sl, s, true);
+}
+
+int tpa_gather(tpa_ctx* ctx, int32_t id, int32_t is_request, void* k_out, void* v_out,
+               void* stream) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  const std::vector<int32_t>* pages;
+  int len;
+  if (is_request) {
+    if (id < 0 || id >= ctx->cfg.max_requests) return fail(TPA_ERR_INVALID_ARG, "request id %d", id);
+    if (!ctx->reqs[id].open) return fail(TPA_ERR_STATE, "request %d is not open", id);
+    pages = &ctx->reqs[id].pages;
+    len = ctx->reqs[id].len;
+  } else {
+    if (id < 0 || id >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", id);
+    const Agent& a = ctx->agents[id];
+    if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", id);
+    if (!a.resident) return fail(TPA_ERR_NOT_RESIDENT, "agent %d is not resident", id);
+    pages = &a.pages;
+    len = a.len;
+  }
+  if (len == 0) return TPA_OK;
+  if (!k_out || !v_out) return fail(TPA_ERR_INVALID_ARG, "null destination");
+  const void* kd = k_out;
+  const void* vd = v_out;
+  if (!ctx->plan_only) {
+    int rc;
+    if ((rc = resolve_host_ptr(k_out, &kd)) || (rc = resolve_host_ptr(v_out, &vd))) return rc;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const uint64_t ready = is_request ? 0 : ctx->agents[id].ready_seq;
+  const int rc = page_copy_call(ctx, *pages, len, 0, nullptr, nullptr, const_cast<void*>(kd),
+                                const_cast<void*>(vd), s, true, ready, nullptr);
+  if (rc) return rc;
+  if (is_request) ctx->reqs[id].last_use = ctx->seq;
+  else ctx->agents[id].last_use = ctx->seq;
+  return TPA_OK;
+}
+
+int tpa_query(tpa_ctx* ctx, int32_t what, int32_t id, int64_t* value) {
+  if (!ctx || !value) return fail(TPA_ERR_INVALID_ARG, "null argument");
+  switch (what) {
+    case TPA_Q_FREE_PAGES: *value = free_count(ctx); return TPA_OK;
+    case TPA_Q_PREFIX_LEN:
+    case TPA_Q_PREFIX_RESIDENT:
+    case TPA_Q_PAGE_OF:
+      if (id < 0 || id >= ctx->cfg.max_agents) return fail(TPA_ERR_INVALID_ARG, "agent id %d", id);
+      if (what == TPA_Q_PREFIX_LEN) *value = ctx->agents[id].len;
+      else if (what == TPA_Q_PREFIX_RESIDENT)
+        *value = ctx->agents[id].len < 0 ? -1 : (ctx->agents[id].resident ? 1 : 0);
+      else
+        *value = ctx->agents[id].pages.empty() ? -1 : ctx->agents[id].pages[0];
+      return TPA_OK;
+    case TPA_Q_SUFFIX_LEN:
+      if (id < 0 || id >= ctx->cfg.max_requests) return fail(TPA_ERR_INVALID_ARG, "request id %d", id);
+      *value = ctx->reqs[id].open ? ctx->reqs[id].len : -1;
+      return TPA_OK;
+    case TPA_Q_NUM_SMS: *value = ctx->num_sms; return TPA_OK;
+    case TPA_Q_LAST_DENSE_ITEMS: *value = ctx->last_dense; return TPA_OK;
+    case TPA_Q_LAST_SUFFIX_ITEMS: *value = ctx->last_suffix; return TPA_OK;
+    case TPA_Q_LAST_LAUNCHES: *value = ctx->last_launches; return TPA_OK;
+    default: return fail(TPA_ERR_INVALID_ARG, "unknown query %d", what);
+  }
+}
+
+int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  switch (option) {
+    case TPA_OPT_DECODE_MODE:
+      if (value != 0 && value != 1) return fail(TPA_ERR_INVALID_ARG, "decode mode %lld", (long long)value);
+      ctx->decode_mode = static_cast<int>(value);
+      return TPA_OK;
+    case TPA_OPT_PREFIX_SPLITS:
+      if (value < 0 || value > 1024) return fail(TPA_ERR_INVALID_ARG, "prefix splits %lld", (long long)value);
+      ctx->prefix_splits = static_cast<int>(value);
+      return TPA_OK;
+    case TPA_OPT_SUFFIX_SPLIT_KEYS:
+      if (value < 0 || value % kPage || value > (1 << 20))
+        return fail(TPA_ERR_INVALID_ARG, "split keys must be a multiple of 16");
+      ctx->suffix_split_keys = static_cast<int>(value);
+      return TPA_OK;
+    case TPA_OPT_CONCURRENT:
+      ctx->concurrent = value ? 1 : 0;
+      return TPA_OK;
+    default: return fail(TPA_ERR_INVALID_ARG, "unknown option %d", option);
+  }
+}
+
+int tpa_device_status(tpa_ctx* ctx, void* stream, uint32_t* status) {
+  if (!ctx || !status) return fail(TPA_ERR_INVALID_ARG, "null argument");
+  *status = 0;
+  if (ctx->plan_only) return TPA_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  CUDA_TRY(cudaStreamSynchronize(s));
+  if (ctx->fork_stream) CUDA_TRY(cudaStreamSynchronize(ctx->fork_stream));
+  CUDA_TRY(cudaMemcpy(status, ctx->status, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+  CUDA_TRY(cudaMemset(ctx->status, 0, sizeof(uint32_t)));
+  if (*status & (kStatusDenseTimeout | kStatusSuffixTimeout))
+    return fail(TPA_ERR_TIMEOUT, "a device-side wait timed out (status 0x%x)", *status);
+  return TPA_OK;
+}
+
+}  // extern "C"
+
+namespace tpa {
+cudaError_t init_kernels() {
+  static bool done = false;
+  if (done) return cudaSuccess;
+  cudaError_t e = init_dense_kernels();
+  if (e != cudaSuccess) return e;
+  e = init_suffix_kernels();
+  if (e == cudaSuccess) done = true;
+  return e;
+}
+}  // namespace tpa

@@ -1,0 +1,113 @@
+// KV writes into the paged pool and page-run copies.
+//
+//  * append: the new tokens of a call (decode tokens, prefill chunks, plain
+//    appends) go to (page, slot) positions chosen by the host planner.
+//    Suffixes start on a fresh page, so shared prefix pages are never
+//    written by a request (the prefix is paid once per agent, Eq. 2).
+//  * page copy: a contiguous [len][Hkv][d] prefix <-> its page run.  This is
+//    the prefix movement between CPU and GPU memory (Sec. IV-B, Eq. 7):
+//    with a mapped pinned-host source it is the reload scatter, with a
+//    pinned-host destination the offload gather.  Host memory is read or
+//    written directly by the kernel over the CPU-GPU link, so a fragmented
+//    (permuted) page run costs no extra copies.
+// Every copy moves 16-byte units; consecutive threads take consecutive
+// units of one token row, so both sides are coalesced.
+#include "kernels.h"
+
+namespace tpa {
+
+namespace {
+
+constexpr int kCopyThreads = 256;
+
+__global__ void __launch_bounds__(kCopyThreads)
+    append_kernel(const AppendRow* __restrict__ rows, int n_rows, const uint4* __restrict__ k_src,
+                  const uint4* __restrict__ v_src, uint4* __restrict__ k_pool,
+                  uint4* __restrict__ v_pool, int64_t num_pages, int hkv, int cpr,
+                  uint32_t* status) {
+  const int64_t total = static_cast<int64_t>(n_rows) * hkv * cpr;
+  for (int64_t u = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; u < total;
+       u += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int c = static_cast<int>(u % cpr);
+    const int64_t t = u / cpr;
+    const int h = static_cast<int>(t % hkv);
+    const int row = static_cast<int>(t / hkv);
+    const AppendRow r = rows[row];
+    if (r.page < 0 || r.page >= num_pages || r.slot < 0 || r.slot >= kPage) {
+      atomicOr(status, kStatusBadPage);
+      continue;
+    }
+    const int64_t src = (static_cast<int64_t>(r.src) * hkv + h) * cpr + c;
+    const int64_t dst = ((static_cast<int64_t>(r.page) * hkv + h) * kPage + r.slot) * cpr + c;
+    k_pool[dst] = k_src[src];
+    v_pool[dst] = v_src[src];
+  }
+}
+
+__global__ void __launch_bounds__(kCopyThreads)
+    page_copy_kernel(const int32_t* __restrict__ pages, int len, int to_pages,
+                     const uint4* __restrict__ k_lin, const uint4* __restrict__ v_lin,
+                     uint4* __restrict__ k_lin_out, uint4* __restrict__ v_lin_out,
+                     uint4* __restrict__ k_pool, uint4* __restrict__ v_pool, int64_t num_pages,
+                     int hkv, int cpr, uint32_t* status) {
+  const int64_t total = static_cast<int64_t>(len) * hkv * cpr;
+  for (int64_t u = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; u < total;
+       u += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int c = static_cast<int>(u % cpr);
+    const int64_t t = u / cpr;
+    const int h = static_cast<int>(t % hkv);
+    const int tok = static_cast<int>(t / hkv);
+    const int64_t page = pages[tok / kPage];
+    if (page < 0 || page >= num_pages) {
+      atomicOr(status, kStatusBadPage);
+      continue;
+    }
+    const int64_t lin = (static_cast<int64_t>(tok) * hkv + h) * cpr + c;
+    const int64_t pg = ((page * hkv + h) * kPage + tok % kPage) * cpr + c;
+    if (to_pages) {
+      k_pool[pg] = k_lin[lin];
+      v_pool[pg] = v_lin[lin];
+    } else {
+      k_lin_out[lin] = k_pool[pg];
+      v_lin_out[lin] = v_pool[pg];
+    }
+  }
+}
+
+int copy_grid(int64_t units) {
+  int64_t blocks = (units + kCopyThreads - 1) / kCopyThreads;
+  if (blocks > 4096) blocks = 4096;
+  if (blocks < 1) blocks = 1;
+  return static_cast<int>(blocks);
+}
+
+}  // namespace
+
+cudaError_t launch_append(const AppendRow* rows, int n_rows, const void* k_src,
+                          const void* v_src, const PoolGeom& pool, uint32_t* status,
+                          cudaStream_t stream) {
+  if (n_rows <= 0) return cudaSuccess;
+  const int cpr = pool.d / 8;
+  const int64_t units = static_cast<int64_t>(n_rows) * pool.hkv * cpr;
+  append_kernel<<<copy_grid(units), kCopyThreads, 0, stream>>>(
+      rows, n_rows, static_cast<const uint4*>(k_src), static_cast<const uint4*>(v_src),
+      static_cast<uint4*>(pool.k), static_cast<uint4*>(pool.v), pool.num_pages, pool.hkv, cpr,
+      status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_page_copy(const int32_t* pages, int len, int to_pages, const void* k_lin,
+                             const void* v_lin, void* k_lin_out, void* v_lin_out,
+                             const PoolGeom& pool, uint32_t* status, cudaStream_t stream) {
+  if (len <= 0) return cudaSuccess;
+  const int cpr = pool.d / 8;
+  const int64_t units = static_cast<int64_t>(len) * pool.hkv * cpr;
+  page_copy_kernel<<<copy_grid(units), kCopyThreads, 0, stream>>>(
+      pages, len, to_pages, static_cast<const uint4*>(k_lin), static_cast<const uint4*>(v_lin),
+      static_cast<uint4*>(k_lin_out), static_cast<uint4*>(v_lin_out),
+      static_cast<uint4*>(pool.k), static_cast<uint4*>(pool.v), pool.num_pages, pool.hkv, cpr,
+      status);
+  return cudaGetLastError();
+}
+
+}  // namespace tpa

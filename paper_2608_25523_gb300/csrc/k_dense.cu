@@ -1,0 +1,440 @@
+// Dense tensor-core attention over paged KV (tcgen05 + TMEM + TMA).
+//
+// Level 1 of the decode cascade.  All requests of agent a share the same
+// resident prefix (Sec. I: one static path of the prefix cache per agent;
+// Sec. III, Eq. 2: the prefix is paid once per agent), so the queries of
+// all of a's decode tokens are stacked into 128-row tiles (128/G tokens x G
+// heads of one kv head) and the prefix K/V is streamed through the tensor
+// cores once per tile instead of once per request.  The same kernel runs
+// chunked causal prefill (Sec. VI cites chunked prefill): a tile of one
+// request's chunk attends to the whole prefix and then causally to the
+// request's own suffix.
+//
+// One CTA = one work item (a 128-row Q tile against up to two key segments).
+//   warp 0      TMA producer: K and V tiles (8 pages x 64-dim boxes, 128B
+//               swizzle) into a 2-stage ring, per-page page-id lookup
+//   warp 1      TMEM owner; one lane issues tcgen05.mma:
+//                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
+//                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
+//               QK of tile j+1 is issued before PV of tile j, so the
+//               softmax of j+1 overlaps the tensor work of j
+//   warps 2..5  softmax: one thread per row reads S from TMEM, masks, keeps
+//               the running max/sum in base 2, writes P (bf16) to shared
+//               memory, rescales O in TMEM only when the max grew by more
+//               than 2^8 (otherwise the stale max stays the reference, which
+//               is exact: the max is only a stabiliser), then the epilogue.
+// Every mbarrier wait is bounded; on a timeout the CTA records a status bit,
+// drains its copies and MMAs, frees TMEM and returns.
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace tpa {
+
+namespace {
+
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+template <int D>
+struct DenseCfg {
+  static constexpr int NCH = D / 64;               // 64-dim chunks of a 128-byte row
+  static constexpr int kChunk = 128 * 128;         // one chunk of a 128-row/128-key tile
+  static constexpr int kQBytes = NCH * kChunk;     // Q   [chunk][row][128 B]
+  static constexpr int kPBytes = 2 * kChunk;       // P   [key chunk][row][128 B]
+  static constexpr int kKVBytes = NCH * kChunk;    // K,V [chunk][key][128 B]
+  static constexpr int kStages = 2;
+  static constexpr int kOffQ = 0;
+  static constexpr int kOffP = kOffQ + kQBytes;
+  static constexpr int kOffK = kOffP + kPBytes;
+  static constexpr int kOffV = kOffK + kStages * kKVBytes;
+  static constexpr int kOffBar = kOffV + kStages * kKVBytes;
+  static constexpr int kNumBars = 16;
+  static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+  static constexpr int kSmem = 1024 + kOffMisc + 64;
+  static constexpr uint32_t kTmemCols = 512;
+  static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
+};
+
+// barrier slots
+enum { B_KFULL = 0, B_KEMPTY = 2, B_VFULL = 4, B_VEMPTY = 6, B_SFULL = 8, B_SFREE = 10,
+       B_PFULL = 12, B_OFULL = 13, B_DRAIN = 14 };
+
+struct TileInfo {
+  int key0;     // first key of the tile within its segment
+  int nvalid;   // keys of the tile inside the range (1..128)
+  int causal;
+  int page_off; // page-list index of the tile's first page
+};
+
+__device__ __forceinline__ TileInfo tile_at(const DenseItem& it, int j) {
+  const int t0 = it.seg_k1[0] > it.seg_k0[0] ? (it.seg_k1[0] - it.seg_k0[0] + 127) / 128 : 0;
+  const int seg = j < t0 ? 0 : 1;
+  const int jj = j < t0 ? j : j - t0;
+  TileInfo t;
+  t.key0 = it.seg_k0[seg] + 128 * jj;
+  const int rest = it.seg_k1[seg] - t.key0;
+  t.nvalid = rest < 128 ? rest : 128;
+  t.causal = it.seg_causal[seg];
+  t.page_off = it.seg_pages[seg] + t.key0 / kPage;
+  return t;
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ DenseParams p) {
+  using C = DenseCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kOffBar);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const DenseItem item = p.items[blockIdx.x];
+  const int ntiles = item.n_tiles;
+
+  // ---------------------------------------------------------------- setup
+  if (threadIdx.x == 0) {
+    *abort_flag = 0;
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars[B_KFULL + i], 1);
+      mbar_init(&bars[B_KEMPTY + i], 1);
+      mbar_init(&bars[B_VFULL + i], 1);
+      mbar_init(&bars[B_VEMPTY + i], 1);
+      mbar_init(&bars[B_SFULL + i], 1);
+      mbar_init(&bars[B_SFREE + i], 128);
+    }
+    mbar_init(&bars[B_PFULL], 128);
+    mbar_init(&bars[B_OFULL], 1);
+    mbar_init(&bars[B_DRAIN], 1);
+    fence_mbar_init();
+    prefetch_tmap(&p.tmap_k);
+    prefetch_tmap(&p.tmap_v);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
+
+  // softmax warps: row of this thread, its token, and the Q row into smem
+  const int row = 32 * (warp & 3) + lane;
+  const int tok = row / G;
+  const bool row_valid = warp >= 2 && tok < item.n_tok;
+  DenseTok dt = {0, 0x7fffffff, 0, 0};
+  if (row_valid) dt = p.toks[item.tok_base + tok];
+  const int head = item.kv_head * G + row % G;
+  if (warp >= 2) {
+    uint8_t* qs = smem + C::kOffQ;
+    const uint4* src = reinterpret_cast<const uint4*>(
+        p.q + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D);
+#pragma unroll
+    for (int u = 0; u < D / 8; ++u) {
+      const uint4 v = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(qs + (u >> 3) * C::kChunk + swz128(row, u & 7)) = v;
+    }
+    fence_proxy_async();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
+      bool pok = true;
+      for (int j = 0; j < ntiles; ++j) {
+        const TileInfo t = tile_at(item, j);
+        const int s = j & 1;
+        const uint32_t ph = (j >> 1) & 1;
+        const int npg = (t.nvalid + kPage - 1) / kPage;
+        const uint32_t bytes = static_cast<uint32_t>(npg * C::NCH * 2048);
+        int z[8];
+        for (int i = 0; i < npg; ++i) {
+          int64_t pid = p.pages[t.page_off + i];
+          if (pid < 0 || pid >= p.num_pages) {
+            atomicOr(p.status, kStatusBadPage);
+            pid = 0;
+          }
+          z[i] = static_cast<int>(pid * p.hkv + item.kv_head);
+        }
+        if (!mbar_wait(&bars[B_KEMPTY + s], ph ^ 1u, abort_flag)) { pok = false; break; }
+        mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
+        uint8_t* kst = smem + C::kOffK + s * C::kKVBytes;
+        for (int i = 0; i < npg; ++i)
+#pragma unroll
+          for (int c = 0; c < C::NCH; ++c)
+            tma_load_3d(kst + c * C::kChunk + i * 2048, &p.tmap_k, &bars[B_KFULL + s], c * 64, 0,
+                        z[i]);
+        kph_last[s] = static_cast<int>(ph);
+        if (!mbar_wait(&bars[B_VEMPTY + s], ph ^ 1u, abort_flag)) { pok = false; break; }
+        mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
+        uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
+        for (int i = 0; i < npg; ++i)
+#pragma unroll
+          for (int c = 0; c < C::NCH; ++c)
+            tma_load_3d(vst + c * C::kChunk + i * 2048, &p.tmap_v, &bars[B_VFULL + s], c * 64, 0,
+                        z[i]);
+        vph_last[s] = static_cast<int>(ph);
+      }
+      if (!pok) {
+        *abort_flag = 1;
+        atomicOr(p.status, kStatusDenseTimeout);
+      }
+      if (*abort_flag) {
+        // let every issued copy land before the CTA's shared memory goes away
+        volatile int never = 0;
+        for (int s = 0; s < 2; ++s) {
+          if (kph_last[s] >= 0) (void)mbar_wait(&bars[B_KFULL + s], kph_last[s], &never);
+          if (vph_last[s] >= 0) (void)mbar_wait(&bars[B_VFULL + s], vph_last[s], &never);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_qk = umma_idesc_bf16(128, 128, false, false);
+      constexpr uint32_t idesc_pv = umma_idesc_bf16(128, D, false, true);
+      const uint32_t qbase = smem_u32(smem + C::kOffQ);
+      const uint32_t pbase = smem_u32(smem + C::kOffP);
+      const uint32_t kbase0 = smem_u32(smem + C::kOffK);
+      const uint32_t vbase0 = smem_u32(smem + C::kOffV);
+      bool ok = true;
+      auto issue_pv = [&](int i) -> bool {
+        const int s = i & 1;
+        if (!mbar_wait(&bars[B_PFULL], i & 1, abort_flag)) return false;
+        if (!mbar_wait(&bars[B_VFULL + s], (i >> 1) & 1, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t vb = vbase0 + s * C::kKVBytes;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t a = umma_sdesc(pbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
+          const uint64_t b = umma_sdesc(vb + kk * 2048, C::kChunk, 1024);
+          umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&bars[B_OFULL]);
+        umma_commit(&bars[B_VEMPTY + s]);
+        return true;
+      };
+      for (int j = 0; j < ntiles && ok; ++j) {
+        const int s = j & 1;
+        const uint32_t ph = (j >> 1) & 1;
+        if (!mbar_wait(&bars[B_KFULL + s], ph, abort_flag) ||
+            !mbar_wait(&bars[B_SFREE + s], ph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kb = kbase0 + s * C::kKVBytes;
+        const uint32_t scol = s ? C::kColS1 : C::kColS0;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint64_t a = umma_sdesc(qbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
+          const uint64_t b = umma_sdesc(kb + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
+          umma_bf16_ss(tmem + scol, a, b, idesc_qk, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&bars[B_SFULL + s]);
+        umma_commit(&bars[B_KEMPTY + s]);
+        if (j > 0) ok = issue_pv(j - 1);
+      }
+      if (ok && ntiles > 0) ok = issue_pv(ntiles - 1);
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(p.status, kStatusDenseTimeout);
+      }
+      // all MMAs issued by this thread complete before TMEM is released
+      umma_commit(&bars[B_DRAIN]);
+      volatile int never = 0;
+      (void)mbar_wait(&bars[B_DRAIN], 0, &never);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax
+    const uint32_t lane_base = static_cast<uint32_t>(32 * (warp & 3)) << 16;
+    const float sc = p.scale_log2;
+    uint8_t* ps = smem + C::kOffP;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    // warp-uniform outcome, so .sync.aligned tcgen05 ops never see a split warp
+    auto wait_all = [&](uint64_t* bar, uint32_t parity) {
+      return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
+    };
+    for (int j = 0; j < ntiles; ++j) {
+      const TileInfo t = tile_at(item, j);
+      const int s = j & 1;
+      if (!wait_all(&bars[B_SFULL + s], (j >> 1) & 1)) { ok = false; break; }
+      tc_fence_after();
+      float x[128];
+      const uint32_t scol = tmem + lane_base + (s ? C::kColS1 : C::kColS0);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(scol + 32 * c, x + 32 * c);
+      tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(&bars[B_SFREE + s]);
+
+      int lim = t.nvalid;
+      if (t.causal && dt.causal_pos < t.key0 + lim) {
+        const int c = dt.causal_pos - t.key0 + 1;
+        lim = c > 0 ? c : 0;
+      }
+      float mx = -INFINITY;
+#pragma unroll
+      for (int n = 0; n < 128; ++n) {
+        x[n] = n < lim ? x[n] * sc : -INFINITY;
+        mx = fmaxf(mx, x[n]);
+      }
+      const float m_new = fmaxf(m_run, mx);
+      const bool grow = m_new > m_run + kRescaleThreshold;
+      const float m_use = grow ? m_new : m_run;
+      const float alpha = grow ? fast_exp2(m_run - m_use) : 1.f;
+      const float mref = m_use == -INFINITY ? 0.f : m_use;
+      float rsum = 0.f;
+#pragma unroll
+      for (int n = 0; n < 128; ++n) {
+        x[n] = fast_exp2(x[n] - mref);
+        rsum += x[n];
+      }
+      if (j > 0) {
+        if (!wait_all(&bars[B_OFULL], (j - 1) & 1)) { ok = false; break; }
+        tc_fence_after();
+        // rescale O rows whose reference max moved (with real content)
+        const bool need = grow && m_run > -INFINITY;
+        if (__any_sync(0xffffffffu, need)) {
+#pragma unroll 1
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld32(tmem + lane_base + C::kColO + 32 * c, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tmem_st32(tmem + lane_base + C::kColO + 32 * c, o);
+          }
+          tmem_wait_st();
+        }
+      }
+      l_run = l_run * alpha + rsum;
+      m_run = m_use;
+      if (t.nvalid < 128) {
+        // keys past the range: zero their V rows (stale data may not be finite)
+        if (!wait_all(&bars[B_VFULL + s], (j >> 1) & 1)) { ok = false; break; }
+        if (row >= t.nvalid) {
+          uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
+#pragma unroll
+          for (int c = 0; c < C::NCH; ++c)
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+              *reinterpret_cast<uint4*>(vst + c * C::kChunk + swz128(row, u)) =
+                  make_uint4(0, 0, 0, 0);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        uint4 v;
+        v.x = pack_bf16(x[8 * u + 0], x[8 * u + 1]);
+        v.y = pack_bf16(x[8 * u + 2], x[8 * u + 3]);
+        v.z = pack_bf16(x[8 * u + 4], x[8 * u + 5]);
+        v.w = pack_bf16(x[8 * u + 6], x[8 * u + 7]);
+        *reinterpret_cast<uint4*>(ps + (u >> 3) * C::kChunk + swz128(row, u & 7)) = v;
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      mbar_arrive(&bars[B_PFULL]);
+    }
+    if (ok && ntiles > 0) {
+      ok = wait_all(&bars[B_OFULL], (ntiles - 1) & 1);
+      if (ok) {
+        tc_fence_after();
+        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tmem + lane_base + C::kColO + 32 * c, o);
+          tmem_wait_ld();
+          if (row_valid) {
+            if (item.out_mode == 0) {
+              const int64_t slot =
+                  dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
+              float4* dst = reinterpret_cast<float4*>(p.part_o + slot * D + 32 * c);
+#pragma unroll
+              for (int i = 0; i < 8; ++i)
+                dst[i] = make_float4(o[4 * i] * inv, o[4 * i + 1] * inv, o[4 * i + 2] * inv,
+                                     o[4 * i + 3] * inv);
+            } else {
+              uint4* dst = reinterpret_cast<uint4*>(
+                  p.out + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D + 32 * c);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                uint4 v;
+                v.x = pack_bf16(o[8 * i + 0] * inv, o[8 * i + 1] * inv);
+                v.y = pack_bf16(o[8 * i + 2] * inv, o[8 * i + 3] * inv);
+                v.z = pack_bf16(o[8 * i + 4] * inv, o[8 * i + 5] * inv);
+                v.w = pack_bf16(o[8 * i + 6] * inv, o[8 * i + 7] * inv);
+                dst[i] = v;
+              }
+            }
+          }
+        }
+        if (row_valid) {
+          const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : -INFINITY;
+          if (item.out_mode == 0) {
+            const int64_t slot = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
+            p.part_lse[slot] = lse;
+          } else {
+            p.lse[static_cast<int64_t>(dt.q_row) * p.hq + head] = lse;
+          }
+        }
+      }
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      atomicOr(p.status, kStatusDenseTimeout);
+    }
+    tc_fence_before();
+  }
+
+  // ---------------------------------------------------------------- teardown
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
+template <int D, int G>
+cudaError_t launch_dense_t(const DenseParams& p, int n_items, cudaStream_t stream) {
+  dense_kernel<D, G><<<n_items, 192, DenseCfg<D>::kSmem, stream>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_dense(const DenseParams& p, int n_items, int head_dim, int group,
+                         cudaStream_t stream) {
+  if (n_items <= 0) return cudaSuccess;
+  if (head_dim == 128 && group == 4) return launch_dense_t<128, 4>(p, n_items, stream);
+  if (head_dim == 128 && group == 8) return launch_dense_t<128, 8>(p, n_items, stream);
+  if (head_dim == 64 && group == 4) return launch_dense_t<64, 4>(p, n_items, stream);
+  if (head_dim == 64 && group == 8) return launch_dense_t<64, 8>(p, n_items, stream);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t init_dense_kernels() {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(dense_kernel<128, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                DenseCfg<128>::kSmem)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(dense_kernel<128, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                DenseCfg<128>::kSmem)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(dense_kernel<64, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                DenseCfg<64>::kSmem)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(dense_kernel<64, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              DenseCfg<64>::kSmem);
+}
+
+}  // namespace tpa

@@ -1,0 +1,82 @@
+// Host-side launchers of the library's kernels.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "plan.h"
+
+namespace tpa {
+
+// Paged pool geometry: bf16 [num_pages][hkv][16][d].
+struct PoolGeom {
+  void* k;
+  void* v;
+  int64_t num_pages;
+  int hkv;
+  int d;
+};
+
+// K/V writes: one row per token into (page, slot).  k_src/v_src are
+// [rows][hkv][d]; device or mapped pinned-host pointers.
+cudaError_t launch_append(const AppendRow* rows, int n_rows, const void* k_src,
+                          const void* v_src, const PoolGeom& pool, uint32_t* status,
+                          cudaStream_t stream);
+
+// Contiguous [len][hkv][d] <-> the pages of a page run.  to_pages = 1 copies
+// src -> pages (prefix write, reload); 0 copies pages -> dst (gather, offload).
+cudaError_t launch_page_copy(const int32_t* pages, int len, int to_pages, const void* k_lin,
+                             const void* v_lin, void* k_lin_out, void* v_lin_out,
+                             const PoolGeom& pool, uint32_t* status, cudaStream_t stream);
+
+struct DenseParams {
+  CUtensorMap tmap_k;  // 3-D view of the K pool: (d, 16 slots, pages*hkv), 64x16 boxes
+  CUtensorMap tmap_v;
+  const __nv_bfloat16* q;
+  __nv_bfloat16* out;
+  float* lse;
+  float* part_o;
+  float* part_lse;
+  const DenseItem* items;
+  const DenseTok* toks;
+  const int32_t* pages;
+  uint32_t* status;
+  int64_t num_pages;
+  int hq, hkv;
+  float scale_log2;  // log2(e) / sqrt(d)
+};
+
+// Dense tensor-core attention of 128-row query tiles (tcgen05 + TMEM + TMA).
+cudaError_t launch_dense(const DenseParams& p, int n_items, int head_dim, int group,
+                         cudaStream_t stream);
+
+struct SuffixParams {
+  CUtensorMap tmap_k;
+  CUtensorMap tmap_v;
+  const __nv_bfloat16* q;
+  float* part_o;
+  float* part_lse;
+  const SuffixItem* items;
+  const int32_t* pages;
+  uint32_t* queue;     // zeroed work counter
+  uint32_t* status;
+  int64_t num_pages;
+  int n_items;
+  int hq, hkv;
+  float scale_log2;
+};
+
+// Split-KV paged attention of G query rows per warp (warp-level MMA).
+cudaError_t launch_suffix(const SuffixParams& p, int num_sms, int head_dim, int group,
+                          cudaStream_t stream);
+
+// Exact LSE merge of each token's partials into bf16 out and fp32 lse.
+cudaError_t launch_merge(const MergeTok* toks, int n_tok, const float* part_o,
+                         const float* part_lse, __nv_bfloat16* out, float* lse, int hq, int d,
+                         cudaStream_t stream);
+
+// Raise dynamic shared-memory limits of the kernels (once per device).
+cudaError_t init_kernels();
+
+}  // namespace tpa

@@ -1,0 +1,80 @@
+// Work-list records built by the host planner and read by the kernels.
+// One call's plan is a single blob uploaded with one host-to-device copy.
+#pragma once
+#include <stdint.h>
+
+namespace tpa {
+
+constexpr int kPage = 16;          // tokens per page
+constexpr int kTileRows = 128;     // query rows of a dense (tensor-core) tile
+constexpr int kTileKeys = 128;     // keys per dense tile (8 pages)
+
+// Status bits of the device status word.
+constexpr uint32_t kStatusDenseTimeout = 1u;
+constexpr uint32_t kStatusSuffixTimeout = 2u;
+constexpr uint32_t kStatusBadPage = 4u;
+
+// One token row of a KV write: row `src` of the source K/V arrays goes to
+// slot `slot` of page `page`.
+struct AppendRow {
+  int32_t src;
+  int32_t page;
+  int32_t slot;
+  int32_t pad;
+};
+
+// Per-token data of a dense tile.
+struct DenseTok {
+  int32_t q_row;       // row of q / out / lse ([rows][Hq][d])
+  int32_t causal_pos;  // causal segment: key index k visible iff k <= causal_pos
+  int32_t slot_base;   // partial slot of (token, head 0, split 0)
+  int32_t n_slots;     // splits per (token, head); slot = slot_base + head * n_slots + split
+};
+
+// One 128-row query tile (128/G tokens x G heads of one kv head) against up
+// to two key segments, each a run of pages of one prefix or one suffix.
+struct DenseItem {
+  int32_t tok_base;       // first DenseTok of the tile
+  int32_t n_tok;          // tokens in the tile (<= 128 / G)
+  int32_t kv_head;
+  int32_t split;          // split index for partial slots (out_mode 0)
+  int32_t out_mode;       // 0: fp32 partial (o, lse); 1: bf16 out + fp32 lse
+  int32_t n_tiles;        // total key tiles over both segments
+  int32_t seg_pages[2];   // offset in the page list of the segment's page 0
+  int32_t seg_k0[2];      // first key of the range (multiple of 16)
+  int32_t seg_k1[2];      // one past the last key of the range (k1 == k0: empty)
+  int32_t seg_causal[2];  // 1: causal mask on this segment
+  int32_t pad[2];
+};
+static_assert(sizeof(DenseItem) == 64, "DenseItem layout");
+
+// One warp of the split-KV kernel: the G query rows of one token against a
+// key range of one page run (a request suffix, or a prefix in flat mode).
+struct SuffixItem {
+  int32_t q_row;
+  int32_t kv_head;
+  int32_t pages;      // offset in the page list of the range's first page
+  int32_t n_keys;     // keys in the range (>= 1), starting at that page's slot 0
+  int32_t slot_base;  // partial slot of (token, head 0, split 0)
+  int32_t n_slots;
+  int32_t split;
+  int32_t pad;
+};
+static_assert(sizeof(SuffixItem) == 32, "SuffixItem layout");
+
+// LSE merge of all partials of one token (every q head).
+struct MergeTok {
+  int32_t q_row;
+  int32_t slot_base;
+  int32_t n_slots;
+  int32_t pad;
+};
+
+// Header of an uploaded plan blob; offsets in bytes from the blob start.
+struct PlanHeader {
+  int32_t n_pages, n_append, n_dense_tok, n_dense, n_suffix, n_merge;
+  int32_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge;
+  uint32_t queue[4];  // zero on upload: atomic work counters of persistent kernels
+};
+
+}  // namespace tpa

@@ -1,0 +1,255 @@
+"""GPU parity of the CUDA path against the fp64 oracle, through the C ABI.
+
+Small workloads span several tiles and ragged tails: prefixes of 0, 1, 15,
+16, 17, 127, 128, 129 and 1000 tokens; cached suffixes of 0..300 tokens;
+more decode requests per agent than one 128-row tile holds; head_dim 64
+and 128; GQA groups 4 and 8; sequential and permuted (fragmented) pools;
+a "sharp" variant with Q scaled by 8 so the softmax is peaked.  Page-table
+work (append, prefix write, reload, offload, gather) must be bit-exact.
+"""
+import zlib
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_25523_gb300 import binding as B
+from paper_2608_25523_gb300.build import build
+from paper_2608_25523_gb300.session import Session, to_device
+from paper_2608_25523_gb300.workloads import config, sharp, small_case, tensors_numpy
+
+from _util import compare, stack_decode_ref
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    build()
+    B.load()
+
+
+def _bits(x):
+    return x.contiguous().view(torch.int16)
+
+
+def _session(w, **kw):
+    t = tensors_numpy(w)
+    return t, Session(w, to_device(t, "cuda"), **kw)
+
+
+def _check_status(s):
+    assert s.ctx.device_status() == 0
+
+
+DECODE_CASES = {
+    # name: (hq, hkv, d, prefix lens, request agents, cached suffix lens, permuted)
+    "d128_g4_mixed": (8, 2, 128, [0, 1, 129, 1000], [0, 1, 2, 3, 1, 2, 3, 3],
+                      [5, 0, 15, 16, 17, 300, 64, 1], False),
+    "d64_g8_edges": (16, 2, 64, [15, 16, 17, 127, 128], [0, 1, 2, 3, 4, 0, 4],
+                     [1, 16, 31, 32, 33, 200, 7], True),
+    "d128_g8_many": (32, 4, 128, [300], [0] * 20, list(range(0, 200, 10)), False),
+    "d64_g4_two_tiles": (8, 2, 64, [257, 40], [0] * 40 + [1] * 3,
+                         [(7 * i) % 90 for i in range(43)], True),
+}
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
+@pytest.mark.parametrize("name", sorted(DECODE_CASES))
+def test_decode_small(name, mode):
+    hq, hkv, d, plen, agents, ctx, perm = DECODE_CASES[name]
+    w = small_case(zlib.crc32(name.encode()) % 1000, hq=hq, hkv=hkv, d=d, prefix_len=plen, req_agent=agents,
+                   req_ctx=ctx, req_prefill=[0] * len(agents), req_decode=[1] * len(agents),
+                   permute=perm)
+    t, s = _session(w)
+    s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    ref = oracle.workload_decode(w, t)
+    o_ref, l_ref = stack_decode_ref(ref, range(len(ids)))
+    compare(out, lse, o_ref, l_ref, f"{name}/{mode}")
+
+
+@pytest.mark.parametrize("splits", [(1, 16), (3, 48), (0, 0)])
+def test_decode_split_choices_agree(splits):
+    """Any split of the prefix (dense level) and suffix (split-KV level)
+    gives the oracle's result: the LSE merge is exact."""
+    w = small_case(7, hq=8, hkv=2, d=128, prefix_len=[700, 33], req_agent=[0, 0, 1, 0],
+                   req_ctx=[100, 257, 3, 31], req_prefill=[0] * 4, req_decode=[1] * 4)
+    t, s = _session(w)
+    s.ctx.set_option(B.OPT_PREFIX_SPLITS, splits[0])
+    s.ctx.set_option(B.OPT_SUFFIX_SPLIT_KEYS, splits[1])
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(out, lse, o_ref, l_ref, f"splits {splits}")
+
+
+def test_decode_sharp_softmax():
+    w = sharp(small_case(11, hq=8, hkv=2, d=128, prefix_len=[513, 64], req_agent=[0, 1, 0, 1, 0],
+                         req_ctx=[40, 2, 129, 300, 0], req_prefill=[0] * 5, req_decode=[1] * 5))
+    t, s = _session(w)
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "sharp")
+
+
+def test_cascade_equals_flat():
+    """The two-level cascade and the flat split-KV path read the same keys
+    in different groupings; they agree to fp32 reordering noise."""
+    w = small_case(13, hq=32, hkv=8, d=128, prefix_len=[1024, 300],
+                   req_agent=[0] * 12 + [1] * 4, req_ctx=[17 * i + 1 for i in range(16)],
+                   req_prefill=[0] * 16, req_decode=[1] * 16)
+    outs = []
+    for mode in (0, 1):
+        t, s = _session(w)
+        s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+        ids, q, kn, vn = s.decode_inputs()
+        out, lse = s.new_outputs(len(ids))
+        s.decode(ids, q, kn, vn, out, lse)
+        torch.cuda.synchronize()
+        _check_status(s)
+        outs.append((out.float().cpu(), lse.cpu()))
+    assert (outs[0][1] - outs[1][1]).abs().max().item() <= 1e-4
+    assert (outs[0][0] - outs[1][0]).abs().max().item() <= 8e-3
+
+
+PREFILL_CASES = {
+    "d128_g4": (8, 2, 128, [0, 129, 1000], [0, 1, 2, 1, 2], [1, 31, 200, 64, 130], 64),
+    "d64_g8": (16, 2, 64, [17, 128], [0, 1, 1], [33, 15, 150], 48),
+    "d128_g8": (32, 4, 128, [250], [0, 0], [100, 17], 32),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PREFILL_CASES))
+def test_prefill_chunks(name):
+    hq, hkv, d, plen, agents, pf, chunk = PREFILL_CASES[name]
+    n = len(agents)
+    w = small_case(zlib.crc32(name.encode()) % 1000, hq=hq, hkv=hkv, d=d, prefix_len=plen, req_agent=agents,
+                   req_ctx=[0] * n, req_prefill=pf, req_decode=[0] * n, chunk=chunk,
+                   permute=True)
+    t, s = _session(w)
+    for rnd in range(w.prefill_rounds()):
+        chunks, ids, lens, q, k, v = s.prefill_inputs(rnd)
+        out, lse = s.new_outputs(sum(lens))
+        s.prefill(ids, lens, q, k, v, out, lse)
+        torch.cuda.synchronize()
+        _check_status(s)
+        row = 0
+        for r, off, c in chunks:
+            o_ref, l_ref = oracle.workload_prefill_chunk(w, t, r, off, c)
+            compare(out[row:row + c], lse[row:row + c], o_ref, l_ref, f"{name} r{r} off{off}")
+            row += c
+
+
+def test_tiny_workload_prefill_then_decode():
+    """The tiny workload: 1 agent, 256-token prefix, 4 requests prefill a
+    64-token suffix in one chunk, then take one decode step."""
+    w = config(0)
+    t, s = _session(w)
+    chunks, ids, lens, q, k, v = s.prefill_inputs(0)
+    out, lse = s.new_outputs(sum(lens))
+    s.prefill(ids, lens, q, k, v, out, lse)
+    torch.cuda.synchronize()
+    row = 0
+    for r, off, c in chunks:
+        o_ref, l_ref = oracle.workload_prefill_chunk(w, t, r, off, c)
+        compare(out[row:row + c], lse[row:row + c], o_ref, l_ref, f"tiny prefill r{r}")
+        row += c
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "tiny decode")
+
+
+# ---------------------------------------------------------------- pages --
+
+@pytest.mark.parametrize("perm", [False, True], ids=["sequential", "permuted"])
+def test_page_roundtrip_bit_exact(perm):
+    w = small_case(21, hq=8, hkv=2, d=128, prefix_len=[1, 16, 17, 300, 0],
+                   req_agent=[0, 1, 2, 3, 4, 3], req_ctx=[0, 1, 15, 16, 33, 250],
+                   req_prefill=[0] * 6, req_decode=[1] * 6, permute=perm)
+    t, s = _session(w)
+    td = s.t
+    for a in range(w.num_agents):
+        L = w.prefix_len[a]
+        if L == 0:
+            continue
+        k = torch.empty(L, w.num_kv_heads, w.head_dim, dtype=torch.bfloat16, device="cuda")
+        v = torch.empty_like(k)
+        s.ctx.gather(a, False, k, v)
+        pk, pv = td.prefix(a, w)
+        torch.cuda.synchronize()
+        assert torch.equal(_bits(k), _bits(pk)) and torch.equal(_bits(v), _bits(pv))
+    # a decode step appends one token per request; gathering must show it
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    for r in range(w.num_requests):
+        L = w.req_ctx[r] + 1
+        k = torch.empty(L, w.num_kv_heads, w.head_dim, dtype=torch.bfloat16, device="cuda")
+        v = torch.empty_like(k)
+        s.ctx.gather(r, True, k, v)
+        sk, sv = td.suffix(r, w, 0, L)
+        torch.cuda.synchronize()
+        assert torch.equal(_bits(k), _bits(sk)) and torch.equal(_bits(v), _bits(sv)), r
+    _check_status(s)
+
+
+def test_offload_reload_bit_exact_on_side_stream():
+    w = small_case(23, hq=8, hkv=2, d=128, prefix_len=[333, 48], req_agent=[0, 1, 0],
+                   req_ctx=[20, 5, 77], req_prefill=[0] * 3, req_decode=[1] * 3, permute=True)
+    t, s = _session(w)
+    L = w.prefix_len[0]
+    hk = torch.empty(L, 2, 128, dtype=torch.bfloat16, pin_memory=True)
+    hv = torch.empty_like(hk, pin_memory=True)
+    side = torch.cuda.Stream()
+    ev = torch.cuda.Event()
+    s.ctx.prefix_offload(0, hk, hv, side, ev)
+    ev.synchronize()
+    pk, pv = s.t.prefix(0, w)
+    assert torch.equal(_bits(hk), _bits(pk.cpu())) and torch.equal(_bits(hv), _bits(pv.cpu()))
+    assert s.ctx.query(B.Q_PREFIX_RESIDENT, 0) == 0
+    ev2 = torch.cuda.Event()
+    s.ctx.prefix_reload(0, hk, hv, side, ev2)
+    # decode on the default stream must see the reloaded prefix without a host sync
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "after reload")
+    k = torch.empty(L, 2, 128, dtype=torch.bfloat16, device="cuda")
+    v = torch.empty_like(k)
+    s.ctx.gather(0, False, k, v)
+    torch.cuda.synchronize()
+    assert torch.equal(_bits(k), _bits(pk)) and torch.equal(_bits(v), _bits(pv))
+
+
+def test_reload_rejects_unpinned_host_memory():
+    w = small_case(25, hq=8, hkv=2, d=64, prefix_len=[40], req_agent=[0], req_ctx=[1],
+                   req_prefill=[0], req_decode=[1])
+    t, s = _session(w)
+    s.ctx.prefix_evict(0)
+    hk = torch.zeros(40, 2, 64, dtype=torch.bfloat16)   # pageable
+    with pytest.raises(B.TpaError) as e:
+        s.ctx.prefix_reload(0, hk, hk)
+    assert e.value.code == B.TPA_ERR_INVALID_ARG
+    assert s.ctx.query(B.Q_PREFIX_RESIDENT, 0) == 0
