@@ -1,0 +1,565 @@
+"""Benchmark of shared-prefix paged attention on one GB300 (or N replicas).
+
+Default workload: the Llama-3-8B attention layer decode step (32 q heads,
+8 kv heads, head_dim 128, bf16): 4 agents with 4096-token prefixes, 64
+decode requests (16 per agent) with cached suffixes uniform in 256..1024,
+page size 16.  One step = one tpa_decode call over the 64 requests (plan,
+KV append of the new tokens, stacked-prefix tcgen05 attention, split-KV
+suffix attention, LSE merge), followed by a table-only truncate that drops
+the appended token again so every step sees the same workload.  Four
+independent copies of the workload are cycled so that ~0.94 GB of KV lies
+between two visits of the same bytes (L2 is 129 MB): every step reads HBM.
+
+value  = algorithmic bytes per step (each prefix once, each suffix once,
+         Q, the new tokens' K/V in and out, O and LSE) / device time, GB/s.
+e2e    = the same metric through the public call with host buffers: the
+         step's q / k_new / v_new come from pinned host memory and O / LSE
+         go back, inside the timed region.
+Also reported (rank 0, N=1): the tcgen05 chunked-prefill workload
+(TFLOP/s), the mixed workload (reload + prefill + Zipf decode, ms/step)
+and the Llama-3-70B decode workload (GB/s), each with its own roofline.
+
+Under torchrun every rank runs its own copy on its own GPU (the path has
+no exchange step: replicas only); value aggregates all ranks over the
+slowest rank's time.
+
+--impl reference times the fp64 CPU oracle on this host's cores on a
+bounded sample of the same workload and metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decode KV HBM GB/s (% of peak) + prefill TFLOP/s, tokens/s at 1×GB300"
+COPIES = 4
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d["bf16_tflops"], d.get("bf16_tflops_sustained", d["bf16_tflops"]), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ------------------------------------------------------------ accounting --
+
+def decode_bytes(w, reqs):
+    """Algorithmic HBM bytes of one decode step over `reqs`: each distinct
+    prefix once, each suffix (with the new token) once, Q in, the new
+    tokens' K/V in and into the pool, O and LSE out."""
+    mu = w.kv_bytes_per_token()
+    agents = sorted({w.req_agent[r] for r in reqs})
+    prefix = sum(w.prefix_len[a] for a in agents) * mu
+    suffix = sum(w.req_ctx[r] + w.req_prefill[r] + 1 for r in reqs) * mu
+    n = len(reqs)
+    qo = 2 * n * w.num_q_heads * w.head_dim * 2 + n * w.num_q_heads * 4
+    new = 2 * n * mu
+    return prefix, suffix, prefix + suffix + qo + new
+
+
+def prefill_flops(w, chunks):
+    """Unmasked (query row, key) pairs x 4 d flops of the chunks (QK^T and PV)."""
+    pairs = 0
+    for r, off, c in chunks:
+        lp = w.prefix_len[w.req_agent[r]]
+        # positions off..off+c-1 see lp prefix keys and p+1 suffix keys
+        pairs += c * lp + c * off + c * (c + 1) // 2
+    return pairs * w.num_q_heads * 4 * w.head_dim
+
+
+# ---------------------------------------------------------------- clocks --
+
+class Clocks:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "20", "-i", str(self.index)], stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)  # first sample lands before the timed region starts
+        self.t0 = time.time()
+
+    def stop(self):
+        self.t1 = time.time()
+        time.sleep(0.05)
+        if self.proc:
+            self.proc.terminate()
+            self.proc.wait()
+        self.f.flush()
+        rows = []
+        for line in open(self.f.name):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[5:9]))
+            except (ValueError, IndexError):
+                continue
+        os.unlink(self.f.name)
+        inside = [r for r in rows if self.t0 - 0.05 <= r[0] <= self.t1 + 0.05]
+        if not inside and rows:
+            inside = [min(rows, key=lambda r: abs(r[0] - (self.t0 + self.t1) / 2))]
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i, v in enumerate(r[3]) if v == "Active"})
+        sm = sorted(r[1] for r in inside)
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": reasons, "samples": len(inside)}
+
+
+# ------------------------------------------------------------- our arm ---
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.build import build
+    from paper_2608_25523_gb300.session import Session
+    from paper_2608_25523_gb300.workloads import config, copy_requests, replicate, tensors_torch
+
+    build()
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    hbm_peak, tf_peak, tf_sust, peak_src = peaks()
+
+    base = config(1)
+    w = replicate(base, COPIES)
+    t = tensors_torch(w, dev)
+    s = Session(w, t, device=dev, extra_tokens=16)
+    n = base.num_requests
+    steps = []
+    for c in range(COPIES):
+        reqs = copy_requests(w, COPIES, c)
+        ids, q, kn, vn = s.decode_inputs(reqs)   # decode positions == request ids here
+        out, lse = s.new_outputs(len(ids))
+        lens = [w.req_ctx[r] for r in ids]
+        steps.append((B.i32_array(ids), q, kn, vn, out, lse, B.i32_array(lens)))
+    prefix_b, suffix_b, step_bytes = decode_bytes(w, copy_requests(w, COPIES, 0))
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        ids, q, kn, vn, out, lse, lens = steps[i % COPIES]
+        s.ctx.decode(ids, q, kn, vn, out, lse, stream)
+        s.ctx.request_truncate(ids, lens)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for i in range(args.warmup):
+        step(i)
+    barrier()
+    props = torch.cuda.get_device_properties(dev)
+    clocks = Clocks(f"GPU-{props.uuid}" if getattr(props, "uuid", None) else str(local_rank))
+    if rank == 0:
+        clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.steps):
+        step(args.warmup + i)
+    e1.record(stream)
+    e1.synchronize()
+    ms = e0.elapsed_time(e1)
+    barrier()
+    clk = clocks.stop() if rank == 0 else None
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    launches_per_step = s.ctx.query(B.Q_LAST_LAUNCHES)
+    ms_step = ms / args.steps
+    value = step_bytes * args.steps * world / (ms / 1e3) / 1e9
+    tokens_s = n * args.steps * world / (ms / 1e3)
+    status = s.ctx.device_status()
+
+    # per-kernel device time (CUDA events on each kernel's stream)
+    s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+    s.ctx.kernel_times(reset=True)
+    kt_steps = min(args.steps, 400)
+    for i in range(kt_steps):
+        step(i)
+    torch.cuda.synchronize(dev)
+    kt = s.ctx.kernel_times(reset=True)
+    s.ctx.set_option(B.OPT_KERNEL_TIMING, 0)
+    kbytes = {"split_kv": suffix_b + n * w.num_q_heads * w.head_dim * 2,
+              "dense_tcgen05": prefix_b + n * w.num_q_heads * w.head_dim * 2}
+    share = {k: v[0] for k, v in kt.items() if v[1]}
+    dom = max(("split_kv", "dense_tcgen05"), key=lambda k: share.get(k, 0.0))
+    dom_ms = kt[dom][0] / max(1, kt[dom][1])
+    achieved = kbytes[dom] / (dom_ms / 1e3) / 1e9
+    kernels = {k: {"launches": v[1], "avg_us": round(1e3 * v[0] / v[1], 2) if v[1] else None,
+                   "share": round(v[0] / sum(share.values()), 3) if v[1] else 0.0}
+               for k, v in kt.items() if v[1]}
+
+    # end to end through the public call with host buffers
+    import torch as _t
+    host = []
+    for ids, q, kn, vn, out, lse, lens in steps:
+        hq, hk, hv = (x.cpu().pin_memory() for x in (q, kn, vn))
+        ho = _t.empty(out.shape, dtype=out.dtype, pin_memory=True)
+        hl = _t.empty(lse.shape, dtype=lse.dtype, pin_memory=True)
+        host.append((hq, hk, hv, ho, hl))
+    h2d = sum(x.numel() * x.element_size() for x in host[0][:3])
+    d2h = sum(x.numel() * x.element_size() for x in host[0][3:])
+    e2e_steps = args.steps
+
+    def e2e_step(i):
+        ids, q, kn, vn, out, lse, lens = steps[i % COPIES]
+        hq, hk, hv, ho, hl = host[i % COPIES]
+        q.copy_(hq, non_blocking=True)
+        kn.copy_(hk, non_blocking=True)
+        vn.copy_(hv, non_blocking=True)
+        s.ctx.decode(ids, q, kn, vn, out, lse, stream)
+        ho.copy_(out, non_blocking=True)
+        hl.copy_(lse, non_blocking=True)
+        s.ctx.request_truncate(ids, lens)
+
+    for i in range(args.warmup):
+        e2e_step(i)
+    barrier()
+    e0.record(stream)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    e1.record(stream)
+    e1.synchronize()
+    ms_e2e = e0.elapsed_time(e1)
+    if world > 1:
+        tt = torch.tensor([ms_e2e], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_e2e = float(tt.item())
+    e2e = {"value": round(step_bytes * e2e_steps * world / (ms_e2e / 1e3) / 1e9, 1), "unit": "GB/s",
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+           "ms_per_step": round(ms_e2e / e2e_steps, 4)}
+
+    result = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 Q/K/V, random-init; no model weights)",
+        "config": {"workload": "llama3_8b_decode: Hq=32 Hkv=8 d=128 bf16, 4 agents x 4096-token "
+                               "prefixes, 64 decode requests (16/agent), cached suffixes U[256,1024], "
+                               "page 16, contiguous pages",
+                   "l2": f"inputs larger than L2: {COPIES} copies cycled, "
+                         f"{COPIES * step_bytes / 1e9:.2f} GB between reuses",
+                   "bytes_per_step": step_bytes, "prefix_bytes": prefix_b, "suffix_bytes": suffix_b,
+                   "parallelism": f"replicas x{world}"},
+        "hbm_frac_of_measured": round(value / world / hbm_peak, 4),
+        "hbm_frac_of_8tbs": round(value / world / 8000.0, 4),
+        "tokens_per_s": round(tokens_s, 1),
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1),
+                     "peak": hbm_peak, "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
+                     "peak_source": peak_src, "traffic": None,
+                     "bytes_per_launch": kbytes[dom], "avg_launch_us": round(dom_ms * 1e3, 2)},
+        "kernels": kernels,
+        "e2e": e2e,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk,
+        "device_status": status,
+    }
+    s.ctx.close()
+    del s, t
+    torch.cuda.empty_cache()
+    if rank == 0 and world == 1 and not args.no_extras:
+        result["prefill"] = bench_prefill(args, dev, tf_peak, peak_src)
+        result["decode_70b"] = bench_70b(args, dev, hbm_peak, peak_src)
+        result["mixed"] = bench_mixed(args, dev)
+    if rank == 0 and world == 1 and not args.no_cpu:
+        result["cpu_baseline"] = cpu_baseline(budget_s=20.0)
+    return result
+
+
+def bench_prefill(args, dev, tf_peak, peak_src):
+    """Chunked causal prefill workload: all 512-token chunk rounds of 256
+    new requests over 8 agents' prefixes, timed as one pass."""
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.session import Session
+    from paper_2608_25523_gb300.workloads import config, tensors_torch
+
+    w = config(2)
+    stream = torch.cuda.current_stream(dev)
+
+    def one_pass(kernel_timing=False):
+        t = tensors_torch(w, dev)
+        s = Session(w, t, device=dev, extra_tokens=0)
+        s.ctx.set_option(B.OPT_KERNEL_TIMING, 1 if kernel_timing else 0)
+        rounds = []
+        for rnd in range(w.prefill_rounds()):
+            chunks, ids, lens, q, k, v = s.prefill_inputs(rnd)
+            out, lse = s.new_outputs(sum(lens))
+            rounds.append((chunks, ids, lens, q, k, v, out, lse))
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for chunks, ids, lens, q, k, v, out, lse in rounds:
+            s.prefill(ids, lens, q, k, v, out, lse, stream)
+        e1.record(stream)
+        e1.synchronize()
+        kt = s.ctx.kernel_times(reset=True) if kernel_timing else None
+        st = s.ctx.device_status()
+        s.ctx.close()
+        return e0.elapsed_time(e1), kt, st, rounds
+
+    one_pass()                                  # warm-up (first-touch, clocks)
+    ms, _, st, rounds = one_pass()
+    _, kt, _, _ = one_pass(kernel_timing=True)
+    flops = sum(prefill_flops(w, r[0]) for r in rounds)
+    tokens = sum(sum(r[2]) for r in rounds)
+    dense_ms = kt["dense_tcgen05"][0]
+    ach = flops / (dense_ms / 1e3) / 1e12
+    return {"workload": "chunked_prefill: 8 agents, prefixes U[2048,8192], 256 requests, suffixes "
+                        "U[512,2048] in 512-token chunks (all rounds)",
+            "tflops": round(flops / (ms / 1e3) / 1e12, 1), "ms": round(ms, 3),
+            "tokens_per_s": round(tokens / (ms / 1e3), 1), "flops": flops,
+            "roofline": {"bound": "tensor", "kernel": "dense_tcgen05", "achieved": round(ach, 1),
+                         "peak": tf_peak, "unit": "TFLOP/s", "frac": round(ach / tf_peak, 4),
+                         "peak_source": peak_src, "traffic": None,
+                         "avg_launch_us": round(1e3 * dense_ms / max(1, kt["dense_tcgen05"][1]), 1)},
+            "device_status": st}
+
+
+def bench_70b(args, dev, hbm_peak, peak_src):
+    """Llama-3-70B layer decode: 6 agents x 16384-token prefixes, 512
+    requests, suffixes U[512,4096]; 5.3 GB of KV per step (> 40x L2)."""
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.session import Session
+    from paper_2608_25523_gb300.workloads import config, tensors_torch
+
+    w = config(4)
+    t = tensors_torch(w, dev)
+    s = Session(w, t, device=dev, extra_tokens=16)
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    lens = [w.req_ctx[r] for r in ids]
+    ida, lna = B.i32_array(ids), B.i32_array(lens)
+    stream = torch.cuda.current_stream(dev)
+    prefix_b, suffix_b, step_bytes = decode_bytes(w, ids)
+
+    def step():
+        s.ctx.decode(ida, q, kn, vn, out, lse, stream)
+        s.ctx.request_truncate(ida, lna)
+
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize(dev)
+    k = 20
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(k):
+        step()
+    e1.record(stream)
+    e1.synchronize()
+    ms = e0.elapsed_time(e1) / k
+    s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+    for _ in range(5):
+        step()
+    kt = s.ctx.kernel_times(reset=True)
+    st = s.ctx.device_status()
+    s.ctx.close()
+    gbs = step_bytes / (ms / 1e3) / 1e9
+    return {"workload": "llama3_70b_decode: Hq=64 Hkv=8 d=128, 6 agents x 16384-token prefixes, "
+                        "512 requests, suffixes U[512,4096]",
+            "value": round(gbs, 1), "unit": "GB/s", "ms_per_step": round(ms, 4),
+            "hbm_frac_of_measured": round(gbs / hbm_peak, 4), "hbm_frac_of_8tbs": round(gbs / 8000, 4),
+            "tokens_per_s": round(len(ids) / (ms / 1e3), 1), "bytes_per_step": step_bytes,
+            "kernels": {kk: {"avg_us": round(1e3 * v[0] / v[1], 1), "launches": v[1]}
+                        for kk, v in kt.items() if v[1]},
+            "device_status": st}
+
+
+def bench_mixed(args, dev):
+    """Mixed step: 2 prefixes reloaded from pinned host on a side stream,
+    8 x 1024-token prefill chunks and 256 Zipf-assigned decode requests on
+    a permuted (fragmented) pool."""
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.session import Session
+    from paper_2608_25523_gb300.workloads import config, tensors_torch
+
+    w = config(3)
+    t = tensors_torch(w, dev)
+    s = Session(w, t, device=dev, extra_tokens=16)
+    s.offload_for_reload()
+    stream = torch.cuda.current_stream(dev)
+    side = torch.cuda.Stream(device=dev)
+    chunks, pids, plens, pq, pk, pv = s.prefill_inputs(0)
+    pout, plse = s.new_outputs(sum(plens))
+    dids, dq, dkn, dvn = s.decode_inputs()
+    dout, dlse = s.new_outputs(len(dids))
+    ida = B.i32_array(dids)
+    lna = B.i32_array([w.req_ctx[r] for r in dids])
+    pida = B.i32_array(pids)
+    zeros = B.i32_array([0] * len(pids))
+
+    def step():
+        s.reload(side_stream=side)
+        s.prefill(pida, plens, pq, pk, pv, pout, plse, stream)
+        s.ctx.decode(ida, dq, dkn, dvn, dout, dlse, stream)
+        s.ctx.request_truncate(ida, lna)
+        s.ctx.request_truncate(pida, zeros)
+        for a in w.reload_agents:
+            s.ctx.prefix_evict(a)
+
+    step()
+    torch.cuda.synchronize(dev)
+    k = 10
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(k):
+        step()
+    e1.record(stream)
+    side.synchronize()
+    e1.synchronize()
+    ms = e0.elapsed_time(e1) / k
+    st = s.ctx.device_status()
+    reload_bytes = sum(w.prefix_len[a] for a in w.reload_agents) * w.kv_bytes_per_token()
+    s.ctx.close()
+    return {"workload": "mixed: 16 agents prefixes U[1024,8192], 256 Zipf(1.1) decode requests "
+                        "(suffixes U[256,1024]), 8 x 1024-token prefill chunks, permuted pool, "
+                        "2 prefixes reloaded from pinned host on a side stream",
+            "ms_per_step": round(ms, 4), "decode_tokens_per_s": round(len(dids) / (ms / 1e3), 1),
+            "prefill_flops": prefill_flops(w, chunks), "reload_bytes": reload_bytes,
+            "device_status": st}
+
+
+# ------------------------------------------------------ oracle baseline --
+
+def _blas_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 0) for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return max(n)
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+def cpu_baseline(budget_s=20.0, per_step_s=None, steps=1, warmup=0):
+    """Time the fp64 oracle on this host's cores over a bounded sample of
+    the decode workload.  The sample unit is one (request, kv head): the
+    oracle's decode step for the G query heads of that kv head.  The value
+    scales the step's algorithmic bytes by the fraction of units done."""
+    import oracle
+    from paper_2608_25523_gb300.workloads import config, tensors_numpy
+
+    w = config(1)
+    t = tensors_numpy(w)
+    dec = w.decode_requests()
+    G, hkv = w.group, w.num_kv_heads
+    units = [(i, g) for i in range(len(dec)) for g in range(hkv)]
+    step_bytes = decode_bytes(w, dec)[2]
+
+    def run(us):
+        for i, g in us:
+            r = dec[i]
+            pk, pv = t.prefix(w.req_agent[r], w)
+            n_cached = w.req_ctx[r] + w.req_prefill[r]
+            sk, sv = t.suffix(r, w, 0, n_cached)
+            nk, nv = t.suffix(r, w, n_cached, n_cached + 1)
+            oracle.decode_step(t.q_decode[i, g * G:(g + 1) * G], pk[:, g:g + 1], pv[:, g:g + 1],
+                               sk[:, g:g + 1], sv[:, g:g + 1], nk[0, g:g + 1], nv[0, g:g + 1])
+
+    t0 = time.perf_counter()
+    run(units[:1])
+    one = time.perf_counter() - t0
+    budget = per_step_s if per_step_s is not None else budget_s
+    per = max(1, min(len(units), int(budget / max(one, 1e-6))))
+    total_s, done = 0.0, 0
+    pos = 0
+    for i in range(warmup + steps):
+        sample = [units[(pos + j) % len(units)] for j in range(per)]
+        pos += per
+        t0 = time.perf_counter()
+        run(sample)
+        dt = time.perf_counter() - t0
+        if i >= warmup:
+            total_s += dt
+            done += per
+    value = step_bytes * (done / len(units)) / total_s / 1e9
+    return {"value": round(value, 4), "unit": "GB/s", "cores": _blas_threads(), "kind": "oracle",
+            "sample": f"{per} of {len(units)} (request, kv head) units of one llama3_8b_decode step "
+                      f"per timed step, {steps} step(s); float64 numpy over per-request "
+                      f"materialised KV; value = step bytes x fraction done / time",
+            "seconds": round(total_s, 2)}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    budget_total = 150.0
+    per_step = budget_total / max(1, args.steps + args.warmup)
+    cb = cpu_baseline(per_step_s=per_step, steps=args.steps, warmup=args.warmup)
+    return {"impl": "reference", "metric": METRIC, "value": cb["value"], "unit": "GB/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * cb["seconds"] / args.steps, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": "llama3_8b_decode (bounded sample per step, see cpu_baseline)"},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-extras", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local_rank = int(os.environ.get("LOCAL_RANK", 0))
+    if args.impl == "reference":
+        res = run_reference(args, rank, world)
+        if res is not None:
+            print(json.dumps(res))
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    res = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(res))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

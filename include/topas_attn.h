@@ -85,7 +85,9 @@ typedef struct tpa_config {
   int32_t max_requests;      /* request ids are 0 .. max_requests-1 */
   int32_t max_tokens;        /* most query/KV token rows in one append, prefill or decode call */
   int32_t max_seq_len;       /* longest prefix and longest suffix, in tokens */
-  int32_t max_splits;        /* most partial results per (token, head) in decode; 0 -> 32 */
+  int32_t max_splits;        /* most partial results per (token, head) in decode; 0 -> 32.
+                                The partial-result workspace holds
+                                min(max_tokens, max_requests) * Hq * max_splits slots */
   int32_t flags;             /* TPA_FLAG_* */
   uint64_t page_order_seed;  /* 0: free pages handed out in id order; else a seeded permutation
                                 (a fragmented pool, as after many evictions and reloads) */
@@ -151,6 +153,15 @@ TPA_API int tpa_request_open(tpa_ctx* ctx, int32_t req, int32_t agent);
  * work already queued that reads them).  Errors: INVALID_ARG, STATE. */
 TPA_API int tpa_request_close(tpa_ctx* ctx, int32_t req);
 
+/* Discard the tails of the suffixes of `n` distinct open requests so that
+ * lens[i] tokens remain in request reqs[i] (0 <= lens[i] <= its length;
+ * host arrays).  Pages past ceil(lens[i]/16) return to the free list after
+ * the work already queued that reads them.  This is the table step of
+ * dropping decode KV, as when a preempted request's generated tokens are
+ * discarded (Sec. IV-B, discarded decode work, Eq. 8) or a speculative tail
+ * is rejected.  No device work.  All or nothing.  Errors: INVALID_ARG, STATE. */
+TPA_API int tpa_request_truncate(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* lens);
+
 /* Append KV tokens to the suffixes of `n` distinct open requests.
  * reqs[i], ntok[i] (host arrays): request ids and token counts (>= 0).
  * k_new, v_new: device bf16 [sum ntok][Hkv][d], request i's tokens
@@ -210,10 +221,21 @@ enum {
                                    through the split-KV kernel (a cross-check path) */
   TPA_OPT_PREFIX_SPLITS = 1,    /* decode: key splits per stacked prefix tile; 0 = automatic */
   TPA_OPT_SUFFIX_SPLIT_KEYS = 2,/* split-KV chunk in keys (multiple of 16); 0 = automatic */
-  TPA_OPT_CONCURRENT = 3        /* 1 (default): prefix and suffix kernels overlap on a forked
+  TPA_OPT_CONCURRENT = 3,       /* 1 (default): prefix and suffix kernels overlap on a forked
                                    stream; 0: one after the other on the caller's stream */
+  TPA_OPT_KERNEL_TIMING = 4     /* 1: bracket every kernel with CUDA events (tpa_kernel_times) */
 };
 TPA_API int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value);
+
+/* Per-kernel device time, for profiling.  While TPA_OPT_KERNEL_TIMING is 1
+ * every kernel launch of the library is bracketed by CUDA events on the
+ * stream it runs on.  This call synchronises with those events and returns,
+ * for each kernel kind k < n (0 KV append, 1 dense tensor-core attention,
+ * 2 split-KV attention, 3 LSE merge, 4 page-run copy), the accumulated time
+ * in milliseconds and the number of launches since the last reset
+ * (`reset` != 0 clears the totals after reading).  Errors: INVALID_ARG, CUDA. */
+TPA_API int tpa_kernel_times(tpa_ctx* ctx, int32_t n, double* total_ms, int64_t* launches,
+                             int32_t reset);
 
 /* Synchronise `stream`, then read and clear the device status word.
  * *status = 0 when no kernel reported a problem; otherwise a bit set:

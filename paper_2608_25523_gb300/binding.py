@@ -33,6 +33,9 @@ Q_FREE_PAGES, Q_PREFIX_LEN, Q_PREFIX_RESIDENT, Q_SUFFIX_LEN, Q_NUM_SMS = 0, 1, 2
 Q_LAST_DENSE_ITEMS, Q_LAST_SUFFIX_ITEMS, Q_LAST_LAUNCHES, Q_PAGE_OF = 5, 6, 7, 8
 # tpa_set_option
 OPT_DECODE_MODE, OPT_PREFIX_SPLITS, OPT_SUFFIX_SPLIT_KEYS, OPT_CONCURRENT = 0, 1, 2, 3
+OPT_KERNEL_TIMING = 4
+# kernel kinds of tpa_kernel_times
+KERNEL_NAMES = ["kv_append", "dense_tcgen05", "split_kv", "lse_merge", "page_copy"]
 
 
 class TpaError(RuntimeError):
@@ -62,6 +65,7 @@ _SIGS = {
     "tpa_prefix_offload": (c_int, [c_void_p, c_int32, c_void_p, c_void_p, c_void_p, c_void_p]),
     "tpa_request_open": (c_int, [c_void_p, c_int32, c_int32]),
     "tpa_request_close": (c_int, [c_void_p, c_int32]),
+    "tpa_request_truncate": (c_int, [c_void_p, c_int32, _I32P, _I32P]),
     "tpa_kv_append": (c_int, [c_void_p, c_int32, _I32P, _I32P, c_void_p, c_void_p, c_void_p]),
     "tpa_prefill_chunk": (c_int, [c_void_p, c_int32, _I32P, _I32P, c_void_p, c_void_p,
                                   c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -71,6 +75,8 @@ _SIGS = {
     "tpa_query": (c_int, [c_void_p, c_int32, c_int32, POINTER(c_int64)]),
     "tpa_set_option": (c_int, [c_void_p, c_int32, c_int64]),
     "tpa_device_status": (c_int, [c_void_p, c_void_p, POINTER(c_uint32)]),
+    "tpa_kernel_times": (c_int, [c_void_p, c_int32, POINTER(ctypes.c_double), POINTER(c_int64),
+                                 c_int32]),
     "tpa_last_error": (c_char_p, []),
 }
 
@@ -126,6 +132,8 @@ def _event(e):
 
 
 def _i32(vals):
+    if isinstance(vals, ctypes.Array):
+        return vals
     vals = list(int(v) for v in vals)
     return (c_int32 * max(1, len(vals)))(*vals)
 
@@ -185,6 +193,10 @@ class Context:
     def request_close(self, req):
         return self._check(self.lib.tpa_request_close(self.handle, req))
 
+    def request_truncate(self, reqs, lens):
+        return self._check(self.lib.tpa_request_truncate(self.handle, len(reqs), _i32(reqs),
+                                                         _i32(lens)))
+
     def kv_append(self, reqs, ntok, k_new, v_new, stream=None):
         return self._check(self.lib.tpa_kv_append(self.handle, len(reqs), _i32(reqs), _i32(ntok),
                                                   _ptr(k_new), _ptr(v_new), _stream(stream)))
@@ -211,12 +223,25 @@ class Context:
     def set_option(self, option, value):
         return self._check(self.lib.tpa_set_option(self.handle, option, value))
 
+    def kernel_times(self, reset=False):
+        """{kernel name: (total ms, launches)} accumulated while kernel timing is on."""
+        n = len(KERNEL_NAMES)
+        ms = (ctypes.c_double * n)()
+        cnt = (c_int64 * n)()
+        self._check(self.lib.tpa_kernel_times(self.handle, n, ms, cnt, 1 if reset else 0))
+        return {KERNEL_NAMES[i]: (ms[i], cnt[i]) for i in range(n)}
+
     def device_status(self, stream=None):
         v = c_uint32()
         rc = self.lib.tpa_device_status(self.handle, _stream(stream), ctypes.byref(v))
         if rc not in (TPA_OK, TPA_ERR_TIMEOUT):
             self._check(rc)
         return v.value
+
+
+def i32_array(vals):
+    """Pre-built id array for repeated calls (skips per-call marshalling)."""
+    return _i32(vals)
 
 
 def make_config(*, num_q_heads, num_kv_heads, head_dim, num_pages, max_agents, max_requests,

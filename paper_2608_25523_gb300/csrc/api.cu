@@ -56,6 +56,8 @@ int fail(int code, const char* fmt, ...) {
   } while (0)
 
 constexpr int kRingSlots = 4;
+constexpr int kKernelKinds = 5;  // append, dense, split-KV, merge, page copy
+enum { K_APPEND = 0, K_DENSE = 1, K_SUFFIX = 2, K_MERGE = 3, K_COPY = 4 };
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -152,6 +154,17 @@ struct tpa_ctx {
   int concurrent = 1;
   int64_t last_dense = 0, last_suffix = 0, last_launches = 0;
 
+  // per-kernel event timing (TPA_OPT_KERNEL_TIMING)
+  int timing = 0;
+  struct Pending {
+    int kind;
+    cudaEvent_t a, b;
+  };
+  std::vector<cudaEvent_t> ev_free;
+  std::vector<Pending> pending;
+  double k_ms[kKernelKinds] = {};
+  int64_t k_n[kKernelKinds] = {};
+
   // scratch for planning (reused to avoid allocations)
   std::vector<uint8_t> scratch;
 };
@@ -175,19 +188,26 @@ int64_t max_pages_of(const tpa_config* c) { return cdiv(c->max_seq_len + 1, kPag
 
 int splits_of(const tpa_config* c) { return c->max_splits > 0 ? c->max_splits : 32; }
 
+// Decode batches are at most min(max_tokens, max_requests) requests (ids are
+// distinct); prefill chunks hold at most max_tokens rows.
+int64_t max_batch_requests(const tpa_config* c) {
+  return std::min<int64_t>(c->max_tokens, c->max_requests);
+}
+
 PlanSizes plan_capacity(const tpa_config* c) {
   const int64_t g = c->num_q_heads / c->num_kv_heads;
   const int64_t tpt = kTileRows / g;
   const int64_t T = c->max_tokens;
-  const int64_t A = std::min<int64_t>(c->max_agents, T);
+  const int64_t R = max_batch_requests(c);
+  const int64_t A = std::min<int64_t>(c->max_agents, R);
   const int64_t S = splits_of(c);
   PlanSizes s;
-  s.pages = (T + A) * max_pages_of(c);
+  s.pages = (R + A) * max_pages_of(c);
   s.append = T;
   s.dense_tok = T;
-  s.dense = c->num_kv_heads * ((cdiv(T, tpt) + A) * S + T + cdiv(T, tpt));
-  s.suffix = T * c->num_kv_heads * S;
-  s.merge = T;
+  s.dense = c->num_kv_heads * std::max((cdiv(R, tpt) + A) * S, cdiv(T, tpt) + R);
+  s.suffix = R * c->num_kv_heads * S;
+  s.merge = R;
   return s;
 }
 
@@ -231,6 +251,53 @@ void give_pages(tpa_ctx* ctx, std::vector<int32_t>& pages, uint64_t tag) {
 int64_t free_count(const tpa_ctx* ctx) {
   return static_cast<int64_t>(ctx->free_pages.size() - ctx->free_head);
 }
+
+// Kernel timing: bracket a launch with events on its stream when enabled.
+cudaEvent_t timing_event(tpa_ctx* ctx) {
+  if (!ctx->ev_free.empty()) {
+    cudaEvent_t e = ctx->ev_free.back();
+    ctx->ev_free.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+int resolve_timing(tpa_ctx* ctx) {
+  for (auto& p : ctx->pending) {
+    float ms = 0.f;
+    CUDA_TRY(cudaEventSynchronize(p.b));
+    CUDA_TRY(cudaEventElapsedTime(&ms, p.a, p.b));
+    ctx->k_ms[p.kind] += ms;
+    ctx->k_n[p.kind] += 1;
+    ctx->ev_free.push_back(p.a);
+    ctx->ev_free.push_back(p.b);
+  }
+  ctx->pending.clear();
+  return TPA_OK;
+}
+
+struct KernelTimer {
+  tpa_ctx* ctx;
+  int kind;
+  cudaStream_t s;
+  cudaEvent_t a = nullptr;
+  KernelTimer(tpa_ctx* c, int k, cudaStream_t st) : ctx(c), kind(k), s(st) {
+    if (ctx->timing && !ctx->plan_only) {
+      if (ctx->pending.size() > 8192) resolve_timing(ctx);
+      a = timing_event(ctx);
+      if (a) cudaEventRecord(a, s);
+    }
+  }
+  ~KernelTimer() {
+    if (!a) return;
+    cudaEvent_t b = timing_event(ctx);
+    if (!b) return;
+    cudaEventRecord(b, s);
+    ctx->pending.push_back({kind, a, b});
+  }
+};
 
 // Acquire the next plan slot (host-blocking only if kRingSlots calls are in flight).
 Slot* acquire_slot(tpa_ctx* ctx) {
@@ -320,7 +387,7 @@ const char* tpa_last_error(void) { return g_err.c_str(); }
 size_t tpa_workspace_size(const tpa_config* cfg) {
   if (!valid_shape(cfg) || cfg->max_tokens <= 0 || cfg->max_seq_len <= 0) return 0;
   const PlanLayout lay = layout_of(plan_capacity(cfg));
-  const int64_t slots = static_cast<int64_t>(cfg->max_tokens) * cfg->num_q_heads * splits_of(cfg);
+  const int64_t slots = max_batch_requests(cfg) * cfg->num_q_heads * splits_of(cfg);
   size_t total = kAlign;                                     // status word
   total += kRingSlots * align_up(lay.total, kAlign);         // plan ring
   total += align_up(slots * cfg->head_dim * sizeof(float), kAlign);
@@ -382,7 +449,7 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
 
   const PlanLayout lay = layout_of(plan_capacity(cfg));
   ctx->plan_cap = align_up(lay.total, kAlign);
-  ctx->part_slots = static_cast<int64_t>(cfg->max_tokens) * ctx->hq * ctx->max_splits;
+  ctx->part_slots = max_batch_requests(cfg) * ctx->hq * ctx->max_splits;
 
   if (plan_only) {
     for (auto& s : ctx->ring) s.host = static_cast<uint8_t*>(std::malloc(ctx->plan_cap));
@@ -474,6 +541,8 @@ int tpa_destroy(tpa_ctx* ctx) {
       cudaStreamSynchronize(ctx->fork_stream);
       cudaStreamDestroy(ctx->fork_stream);
     }
+    resolve_timing(ctx);
+    for (cudaEvent_t e : ctx->ev_free) cudaEventDestroy(e);
     if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
     if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
   }
@@ -519,6 +588,7 @@ static int page_copy_call(tpa_ctx* ctx, const std::vector<int32_t>& pages, int l
   int rc = upload(ctx, sl, lay.total, s);
   if (rc) return rc;
   if (!ctx->plan_only) {
+    KernelTimer kt(ctx, K_COPY, s);
     CUDA_TRY(launch_page_copy(dev_ptr<int32_t>(sl, lay.off_pages), len, to_pages, k_in, v_in, k_out,
                               v_out, ctx->pool, ctx->status, s));
   }
@@ -673,6 +743,28 @@ int tpa_request_close(tpa_ctx* ctx, int32_t req) {
   return TPA_OK;
 }
 
+int tpa_request_truncate(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* lens) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  int rc = check_batch(ctx, n, reqs, false);
+  if (rc) return rc;
+  if (!lens) return fail(TPA_ERR_INVALID_ARG, "null lengths");
+  for (int i = 0; i < n; ++i)
+    if (lens[i] < 0 || lens[i] > ctx->reqs[reqs[i]].len)
+      return fail(TPA_ERR_INVALID_ARG, "truncate request %d to %d of %d tokens", reqs[i], lens[i],
+                  ctx->reqs[reqs[i]].len);
+  for (int i = 0; i < n; ++i) {
+    Request& r = ctx->reqs[reqs[i]];
+    const size_t keep = static_cast<size_t>(cdiv(lens[i], kPage));
+    if (r.pages.size() > keep) {
+      std::vector<int32_t> tail(r.pages.begin() + keep, r.pages.end());
+      r.pages.resize(keep);
+      give_pages(ctx, tail, r.last_use);
+    }
+    r.len = lens[i];
+  }
+  return TPA_OK;
+}
+
 // Reserve pages for appending ntok[i] tokens to request reqs[i]; all or nothing.
 static int reserve_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* ntok,
                           uint64_t* tag) {
@@ -733,9 +825,11 @@ int tpa_kv_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* n
   chain_begin(ctx, s);
   wait_for_seq(ctx, tag, s);
   if ((rc = upload(ctx, sl, lay.total, s))) return rc;
-  if (!ctx->plan_only)
+  if (!ctx->plan_only) {
+    KernelTimer kt(ctx, K_APPEND, s);
     CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
                            v_new, ctx->pool, ctx->status, s));
+  }
   for (int i = 0; i < n; ++i) {
     Request& r = ctx->reqs[reqs[i]];
     r.len += ntok[i];
@@ -981,8 +1075,11 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
 
   int launches = 0;
   if (!ctx->plan_only) {
-    CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), n, k_new, v_new, ctx->pool,
-                           ctx->status, s));
+    {
+      KernelTimer kt(ctx, K_APPEND, s);
+      CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), n, k_new, v_new, ctx->pool,
+                             ctx->status, s));
+    }
     ++launches;
     const float scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(ctx->d));
     cudaStream_t ds = s;
@@ -1009,6 +1106,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       dp.hq = hq;
       dp.hkv = hkv;
       dp.scale_log2 = scale_log2;
+      KernelTimer kt(ctx, K_DENSE, ds);
       CUDA_TRY(launch_dense(dp, nd, ctx->d, G, ds));
       ++launches;
     }
@@ -1028,6 +1126,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       sp.hq = hq;
       sp.hkv = hkv;
       sp.scale_log2 = scale_log2;
+      KernelTimer kt(ctx, K_SUFFIX, s);
       CUDA_TRY(launch_suffix(sp, ctx->num_sms, ctx->d, G, s));
       ++launches;
     }
@@ -1035,8 +1134,11 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       CUDA_TRY(cudaEventRecord(ctx->ev_join, ctx->fork_stream));
       CUDA_TRY(cudaStreamWaitEvent(s, ctx->ev_join, 0));
     }
-    CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
-                          static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, s));
+    {
+      KernelTimer kt(ctx, K_MERGE, s);
+      CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
+                            static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, s));
+    }
     ++launches;
   }
   for (int i = 0; i < n; ++i) {
@@ -1160,8 +1262,11 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   for (int32_t a : agents_seen) wait_for_seq(ctx, ctx->agents[a].ready_seq, s);
   if ((rc = upload(ctx, sl, lay.total, s))) return rc;
   if (!ctx->plan_only) {
-    CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
-                           v_new, ctx->pool, ctx->status, s));
+    {
+      KernelTimer kt(ctx, K_APPEND, s);
+      CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
+                             v_new, ctx->pool, ctx->status, s));
+    }
     DenseParams dp{};
     dp.tmap_k = ctx->tmap_k;
     dp.tmap_v = ctx->tmap_v;
@@ -1178,6 +1283,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
     dp.hq = hq;
     dp.hkv = hkv;
     dp.scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(ctx->d));
+    KernelTimer kt(ctx, K_DENSE, s);
     CUDA_TRY(launch_dense(dp, nd, ctx->d, G, s));
   }
   for (int i = 0; i < n; ++i) {
@@ -1273,8 +1379,28 @@ int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
     case TPA_OPT_CONCURRENT:
       ctx->concurrent = value ? 1 : 0;
       return TPA_OK;
+    case TPA_OPT_KERNEL_TIMING:
+      ctx->timing = value ? 1 : 0;
+      return TPA_OK;
     default: return fail(TPA_ERR_INVALID_ARG, "unknown option %d", option);
   }
+}
+
+int tpa_kernel_times(tpa_ctx* ctx, int32_t n, double* total_ms, int64_t* launches, int32_t reset) {
+  if (!ctx || n < 0 || (n > 0 && (!total_ms || !launches)))
+    return fail(TPA_ERR_INVALID_ARG, "bad arguments");
+  int rc = resolve_timing(ctx);
+  if (rc) return rc;
+  for (int k = 0; k < n; ++k) {
+    total_ms[k] = k < kKernelKinds ? ctx->k_ms[k] : 0.0;
+    launches[k] = k < kKernelKinds ? ctx->k_n[k] : 0;
+  }
+  if (reset)
+    for (int k = 0; k < kKernelKinds; ++k) {
+      ctx->k_ms[k] = 0.0;
+      ctx->k_n[k] = 0;
+    }
+  return TPA_OK;
 }
 
 int tpa_device_status(tpa_ctx* ctx, void* stream, uint32_t* status) {

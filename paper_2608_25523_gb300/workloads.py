@@ -263,3 +263,25 @@ def tensors_torch(w: Workload, device) -> Tensors:
     return Tensors(draw(pn, hkv, d), draw(pn, hkv, d), draw(sn, hkv, d), draw(sn, hkv, d),
                    draw(qn, hq, d, scale=w.q_scale), draw(nd, hq, d, scale=w.q_scale),
                    poff, soff, qoff)
+
+
+def replicate(w: Workload, copies: int) -> Workload:
+    """`copies` independent copies of a workload in one pool (agents and
+    requests renumbered per copy).  Cycling a benchmark over the copies keeps
+    the bytes touched between two visits of the same data far above the L2
+    size, so every step reads its KV from HBM."""
+    na, nr = w.num_agents, w.num_requests
+    return replace(
+        w, name=f"{w.name}_x{copies}",
+        prefix_len=list(w.prefix_len) * copies,
+        req_agent=[a + c * na for c in range(copies) for a in w.req_agent],
+        req_ctx=list(w.req_ctx) * copies,
+        req_prefill=list(w.req_prefill) * copies,
+        req_decode=list(w.req_decode) * copies,
+        reload_agents=[a + c * na for c in range(copies) for a in w.reload_agents])
+
+
+def copy_requests(w: Workload, copies: int, c: int) -> list:
+    """Request ids of copy `c` of replicate(w, copies)."""
+    n = w.num_requests // copies
+    return list(range(c * n, (c + 1) * n))

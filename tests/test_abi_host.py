@@ -42,8 +42,9 @@ def test_exports_every_declared_symbol(lib):
 
 def test_workspace_size(lib):
     ok = B.make_config(num_q_heads=32, num_kv_heads=8, head_dim=128, num_pages=10, max_agents=1,
-                       max_requests=1, max_tokens=64, max_seq_len=1000)
-    assert B.workspace_size(ok) > 64 * 32 * 32 * 128 * 4
+                       max_requests=100, max_tokens=64, max_seq_len=1000)
+    # partial results: min(max_tokens, max_requests) x Hq x 32 splits x (d + 1) floats
+    assert B.workspace_size(ok) > 64 * 32 * 32 * 129 * 4
     for hq, hkv, d in [(32, 8, 96), (12, 4, 128), (32, 2, 128)]:
         bad = B.make_config(num_q_heads=hq, num_kv_heads=hkv, head_dim=d, num_pages=10,
                             max_agents=1, max_requests=1, max_tokens=64, max_seq_len=1000)
