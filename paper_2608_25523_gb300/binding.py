@@ -128,6 +128,10 @@ def _event(e):
         return None
     if isinstance(e, int):
         return e
+    if not e.cuda_event:
+        # torch creates the CUDA event lazily on its first record; the library
+        # records it again on the stream of the call
+        e.record()
     return e.cuda_event
 
 
