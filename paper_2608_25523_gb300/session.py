@@ -57,25 +57,25 @@ class Session:
                 ctx.prefix_write(a, k.contiguous(), v.contiguous())
         for r in range(w.num_requests):
             ctx.request_open(r, w.req_agent[r])
-        # cached suffix context, in batches of at most max_tokens rows
-        batch, rows = [], 0
-        for r in range(w.num_requests):
-            c = w.req_ctx[r]
-            if c == 0:
-                continue
-            if rows + c > self.max_tokens and batch:
-                self._append_ctx(batch)
-                batch, rows = [], 0
-            batch.append(r)
-            rows += c
-        if batch:
-            self._append_ctx(batch)
+        # cached suffix context, in calls of at most max_tokens rows (a long
+        # context is split across calls; each call takes a request once)
+        done = [0] * w.num_requests
+        pending = [r for r in range(w.num_requests) if w.req_ctx[r] > 0]
+        while pending:
+            batch, rows = [], 0
+            for r in pending:
+                take = min(w.req_ctx[r] - done[r], self.max_tokens - rows)
+                if take <= 0:
+                    break
+                batch.append((r, done[r], take))
+                rows += take
+            ks, vs = zip(*[t.suffix(r, w, lo, lo + n) for r, lo, n in batch])
+            self.ctx.kv_append([r for r, _, _ in batch], [n for _, _, n in batch],
+                               torch.cat(ks), torch.cat(vs))
+            for r, lo, n in batch:
+                done[r] += n
+            pending = [r for r in pending if done[r] < w.req_ctx[r]]
         torch.cuda.synchronize(self.device)
-
-    def _append_ctx(self, reqs):
-        w, t = self.w, self.t
-        ks, vs = zip(*[t.suffix(r, w, 0, w.req_ctx[r]) for r in reqs])
-        self.ctx.kv_append(reqs, [w.req_ctx[r] for r in reqs], torch.cat(ks), torch.cat(vs))
 
     # ------------------------------------------------------------------ steps
     def decode_inputs(self, reqs=None):
