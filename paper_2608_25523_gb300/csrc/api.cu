@@ -908,7 +908,8 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     if (flat || lp == 0) continue;
     const int64_t tiles = cdiv(lp, kTileKeys);
     int64_t ns = ctx->prefix_splits;
-    if (ns <= 0) ns = std::max<int64_t>(1, cdiv(ctx->num_sms, std::max(1, n_units)));
+    // one wave: at most as many dense CTAs as SMs
+    if (ns <= 0) ns = std::max<int64_t>(1, ctx->num_sms / std::max(1, n_units));
     ns = std::min<int64_t>(ns, tiles);
     g.tiles_per_split = static_cast<int32_t>(cdiv(tiles, ns));
     g.n_split = static_cast<int32_t>(cdiv(tiles, g.tiles_per_split));

@@ -119,8 +119,13 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
     prefetch_tmap(&p.tmap_v);
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
+  tc_fence_before();
+  __syncthreads();  // barriers initialised, TMEM allocated: the producer can start
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
 
   // softmax warps: row of this thread, its token, and the Q row into smem
+  // (overlaps the producer's first K/V loads)
   const int row = 32 * (warp & 3) + lane;
   const int tok = row / G;
   const bool row_valid = warp >= 2 && tok < item.n_tok;
@@ -131,23 +136,37 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
     uint8_t* qs = smem + C::kOffQ;
     const uint4* src = reinterpret_cast<const uint4*>(
         p.q + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D);
+    uint4 v[D / 8];
 #pragma unroll
-    for (int u = 0; u < D / 8; ++u) {
-      const uint4 v = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
-      *reinterpret_cast<uint4*>(qs + (u >> 3) * C::kChunk + swz128(row, u & 7)) = v;
-    }
+    for (int u = 0; u < D / 8; ++u) v[u] = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int u = 0; u < D / 8; ++u)
+      *reinterpret_cast<uint4*>(qs + (u >> 3) * C::kChunk + swz128(row, u & 7)) = v[u];
     fence_proxy_async();
   }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
+  // Q is complete before the MMA warp issues the first QK (softmax warps + MMA warp)
+  if (warp >= 1) asm volatile("bar.sync 1, 160;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
       bool pok = true;
+      auto fetch = [&](int j, int* z) {  // page ids of tile j (0 when past the range)
+        const TileInfo t = tile_at(item, j);
+        const int npg = (t.nvalid + kPage - 1) / kPage;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          int64_t pid = i < npg ? p.pages[t.page_off + i] : 0;
+          if (pid < 0 || pid >= p.num_pages) {
+            atomicOr(p.status, kStatusBadPage);
+            pid = 0;
+          }
+          z[i] = static_cast<int>(pid * p.hkv + item.kv_head);
+        }
+      };
+      int znext[8];
+      if (ntiles > 0) fetch(0, znext);
       for (int j = 0; j < ntiles; ++j) {
         const TileInfo t = tile_at(item, j);
         const int s = j & 1;
@@ -155,14 +174,9 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
         const int npg = (t.nvalid + kPage - 1) / kPage;
         const uint32_t bytes = static_cast<uint32_t>(npg * C::NCH * 2048);
         int z[8];
-        for (int i = 0; i < npg; ++i) {
-          int64_t pid = p.pages[t.page_off + i];
-          if (pid < 0 || pid >= p.num_pages) {
-            atomicOr(p.status, kStatusBadPage);
-            pid = 0;
-          }
-          z[i] = static_cast<int>(pid * p.hkv + item.kv_head);
-        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) z[i] = znext[i];
+        if (j + 1 < ntiles) fetch(j + 1, znext);
         if (!mbar_wait(&bars[B_KEMPTY + s], ph ^ 1u, abort_flag)) { pok = false; break; }
         mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
         uint8_t* kst = smem + C::kOffK + s * C::kKVBytes;
