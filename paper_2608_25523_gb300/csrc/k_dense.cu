@@ -295,23 +295,42 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
         const int c = dt.causal_pos - t.key0 + 1;
         lim = c > 0 ? c : 0;
       }
-      float mx = -INFINITY;
+      if (lim < 128) {
 #pragma unroll
-      for (int n = 0; n < 128; ++n) {
-        x[n] = n < lim ? x[n] * sc : -INFINITY;
-        mx = fmaxf(mx, x[n]);
+        for (int n = 0; n < 128; ++n) x[n] = n < lim ? x[n] : -INFINITY;
       }
+      // row max of the raw scores: 8 independent chains of 3-input max
+      float acc[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] = fmaxf(x[i], x[i + 8]);
+#pragma unroll
+      for (int k = 16; k < 128; k += 16)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], x[k + i], x[k + 8 + i]);
+      const float mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
+                                fmaxf(acc[6], acc[7]));
+      const float mx = mraw * sc;  // sc > 0: max of the scaled scores
       const float m_new = fmaxf(m_run, mx);
       const bool grow = m_new > m_run + kRescaleThreshold;
       const float m_use = grow ? m_new : m_run;
       const float alpha = grow ? fast_exp2(m_run - m_use) : 1.f;
-      const float mref = m_use == -INFINITY ? 0.f : m_use;
-      float rsum = 0.f;
+      const float nref = m_use == -INFINITY ? 0.f : -m_use;
+      // p = 2^(s * sc - m): packed FMAs, then MUFU ex2; 8 independent sum chains
+      float sacc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int n = 0; n < 128; ++n) {
-        x[n] = fast_exp2(x[n] - mref);
-        rsum += x[n];
+      for (int n = 0; n < 128; n += 2) {
+        ffma2(x[n], x[n + 1], x[n], x[n + 1], sc, sc, nref, nref);
+        x[n] = fast_exp2(x[n]);
+        x[n + 1] = fast_exp2(x[n + 1]);
       }
+#pragma unroll
+      for (int n = 0; n < 128; n += 16)
+#pragma unroll
+        for (int i = 0; i < 8; i += 2)
+          fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i], x[n + 2 * i + 1]),
+          fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i + 2], x[n + 2 * i + 3]);
+      const float rsum = ((sacc[0] + sacc[1]) + (sacc[2] + sacc[3])) +
+                         ((sacc[4] + sacc[5]) + (sacc[6] + sacc[7]));
       if (j > 0) {
         if (!wait_all(&bars[B_OFULL], (j - 1) & 1)) { ok = false; break; }
         tc_fence_after();
