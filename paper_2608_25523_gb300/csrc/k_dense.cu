@@ -12,17 +12,21 @@
 //
 // One CTA = one work item (a 128-row Q tile against up to two key segments).
 //   warp 0      TMA producer: K and V tiles (8 pages x 64-dim boxes, 128B
-//               swizzle) into a 2-stage ring, per-page page-id lookup
+//               swizzle) into a 2-stage ring, page ids fetched a tile ahead
 //   warp 1      TMEM owner; one lane issues tcgen05.mma:
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
 //                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
 //               QK of tile j+1 is issued before PV of tile j, so the
 //               softmax of j+1 overlaps the tensor work of j
-//   warps 2..5  softmax: one thread per row reads S from TMEM, masks, keeps
-//               the running max/sum in base 2, writes P (bf16) to shared
-//               memory, rescales O in TMEM only when the max grew by more
-//               than 2^8 (otherwise the stale max stays the reference, which
-//               is exact: the max is only a stabiliser), then the epilogue.
+//   warps 2..9  softmax, two warps per TMEM lane quarter: warp 2+q+4h owns
+//               rows 32q..32q+31 and key half h (64 keys).  Both warps of a
+//               pair compute the full-row max (so their running max agrees
+//               without synchronising), exponentiate their own half in base
+//               2, keep a partial row sum, and write their half of P (bf16)
+//               to shared memory.  O in TMEM is rescaled only when the max
+//               grew by more than 2^8; otherwise the stale max stays the
+//               reference, which is exact (the max is only a stabiliser).
+//               The two partial sums meet once, in the epilogue.
 // Every mbarrier wait is bounded; on a timeout the CTA records a status bit,
 // drains its copies and MMAs, frees TMEM and returns.
 #include "kernels.h"
@@ -34,6 +38,8 @@ namespace {
 
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr int kThreads = 320;               // producer, MMA, 8 softmax warps
+constexpr int kSoftmax = 256;
 
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
@@ -55,7 +61,8 @@ struct DenseCfg {
   static constexpr int kOffV = kOffK + kStages * kKVBytes;
   static constexpr int kOffBar = kOffV + kStages * kKVBytes;
   static constexpr int kNumBars = 16;
-  static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+  static constexpr int kOffL = kOffBar + kNumBars * 8;   // partial row sums [2][128]
+  static constexpr int kOffMisc = kOffL + 2 * 128 * 4;
   static constexpr int kSmem = 1024 + kOffMisc + 64;
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
@@ -86,12 +93,13 @@ __device__ __forceinline__ TileInfo tile_at(const DenseItem& it, int j) {
 }
 
 template <int D, int G>
-__global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ DenseParams p) {
+__global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constant__ DenseParams p) {
   using C = DenseCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kOffBar);
+  float* lpart = reinterpret_cast<float*>(smem + C::kOffL);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
@@ -109,9 +117,9 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
       mbar_init(&bars[B_VFULL + i], 1);
       mbar_init(&bars[B_VEMPTY + i], 1);
       mbar_init(&bars[B_SFULL + i], 1);
-      mbar_init(&bars[B_SFREE + i], 128);
+      mbar_init(&bars[B_SFREE + i], kSoftmax);
     }
-    mbar_init(&bars[B_PFULL], 128);
+    mbar_init(&bars[B_PFULL], kSoftmax);
     mbar_init(&bars[B_OFULL], 1);
     mbar_init(&bars[B_DRAIN], 1);
     fence_mbar_init();
@@ -124,28 +132,33 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  // softmax warps: row of this thread, its token, and the Q row into smem
-  // (overlaps the producer's first K/V loads)
-  const int row = 32 * (warp & 3) + lane;
+  // softmax threads: row, key half, token; their slice of the Q row goes to
+  // shared memory while the producer's first K/V loads are in flight
+  const int sw = warp - 2;                 // softmax warp index 0..7
+  const int half = sw >> 2;                // key half (and O column half)
+  const int row = 32 * (warp & 3) + lane;  // TMEM lane quarter = warp % 4
   const int tok = row / G;
   const bool row_valid = warp >= 2 && tok < item.n_tok;
   DenseTok dt = {0, 0x7fffffff, 0, 0};
   if (row_valid) dt = p.toks[item.tok_base + tok];
   const int head = item.kv_head * G + row % G;
   if (warp >= 2) {
+    constexpr int U = D / 16;  // 16-byte units of this thread's half row
     uint8_t* qs = smem + C::kOffQ;
     const uint4* src = reinterpret_cast<const uint4*>(
-        p.q + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D);
-    uint4 v[D / 8];
+        p.q + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D) + half * U;
+    uint4 v[U];
 #pragma unroll
-    for (int u = 0; u < D / 8; ++u) v[u] = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
+    for (int u = 0; u < U; ++u) v[u] = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
 #pragma unroll
-    for (int u = 0; u < D / 8; ++u)
-      *reinterpret_cast<uint4*>(qs + (u >> 3) * C::kChunk + swz128(row, u & 7)) = v[u];
+    for (int u = 0; u < U; ++u) {
+      const int gu = half * U + u;
+      *reinterpret_cast<uint4*>(qs + (gu >> 3) * C::kChunk + swz128(row, gu & 7)) = v[u];
+    }
     fence_proxy_async();
   }
   // Q is complete before the MMA warp issues the first QK (softmax warps + MMA warp)
-  if (warp >= 1) asm volatile("bar.sync 1, 160;" ::: "memory");
+  if (warp >= 1) asm volatile("bar.sync 1, 288;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -180,20 +193,24 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
         if (!mbar_wait(&bars[B_KEMPTY + s], ph ^ 1u, abort_flag)) { pok = false; break; }
         mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
         uint8_t* kst = smem + C::kOffK + s * C::kKVBytes;
-        for (int i = 0; i < npg; ++i)
 #pragma unroll
-          for (int c = 0; c < C::NCH; ++c)
-            tma_load_3d(kst + c * C::kChunk + i * 2048, &p.tmap_k, &bars[B_KFULL + s], c * 64, 0,
-                        z[i]);
+        for (int i = 0; i < 8; ++i)
+          if (i < npg)
+#pragma unroll
+            for (int c = 0; c < C::NCH; ++c)
+              tma_load_3d(kst + c * C::kChunk + i * 2048, &p.tmap_k, &bars[B_KFULL + s], c * 64,
+                          0, z[i]);
         kph_last[s] = static_cast<int>(ph);
         if (!mbar_wait(&bars[B_VEMPTY + s], ph ^ 1u, abort_flag)) { pok = false; break; }
         mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
         uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
-        for (int i = 0; i < npg; ++i)
 #pragma unroll
-          for (int c = 0; c < C::NCH; ++c)
-            tma_load_3d(vst + c * C::kChunk + i * 2048, &p.tmap_v, &bars[B_VFULL + s], c * 64, 0,
-                        z[i]);
+        for (int i = 0; i < 8; ++i)
+          if (i < npg)
+#pragma unroll
+            for (int c = 0; c < C::NCH; ++c)
+              tma_load_3d(vst + c * C::kChunk + i * 2048, &p.tmap_v, &bars[B_VFULL + s], c * 64,
+                          0, z[i]);
         vph_last[s] = static_cast<int>(ph);
       }
       if (!pok) {
@@ -269,6 +286,8 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
   } else {
     // ------------------------------------------------------------ softmax
     const uint32_t lane_base = static_cast<uint32_t>(32 * (warp & 3)) << 16;
+    const int own = half * 64;   // first S column of this thread's key half
+    const int other = 64 - own;
     const float sc = p.scale_log2;
     uint8_t* ps = smem + C::kOffP;
     float m_run = -INFINITY, l_run = 0.f;
@@ -282,10 +301,12 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
       const int s = j & 1;
       if (!wait_all(&bars[B_SFULL + s], (j >> 1) & 1)) { ok = false; break; }
       tc_fence_after();
-      float x[128];
       const uint32_t scol = tmem + lane_base + (s ? C::kColS1 : C::kColS0);
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(scol + 32 * c, x + 32 * c);
+      float x[64], y[64];
+      tmem_ld32(scol + own, x);
+      tmem_ld32(scol + own + 32, x + 32);
+      tmem_ld32(scol + other, y);
+      tmem_ld32(scol + other + 32, y + 32);
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(&bars[B_SFREE + s]);
@@ -297,16 +318,21 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
       }
       if (lim < 128) {
 #pragma unroll
-        for (int n = 0; n < 128; ++n) x[n] = n < lim ? x[n] : -INFINITY;
+        for (int n = 0; n < 64; ++n) {
+          x[n] = own + n < lim ? x[n] : -INFINITY;
+          y[n] = other + n < lim ? y[n] : -INFINITY;
+        }
       }
-      // row max of the raw scores: 8 independent chains of 3-input max
+      // full-row max of the raw scores: 8 independent chains of 3-input max
       float acc[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) acc[i] = fmaxf(x[i], x[i + 8]);
+      for (int i = 0; i < 8; ++i) acc[i] = fmax3f(x[i], x[i + 8], y[i]);
 #pragma unroll
-      for (int k = 16; k < 128; k += 16)
+      for (int k = 16; k < 64; k += 8)
 #pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], x[k + i], x[k + 8 + i]);
+        for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], x[k + i], y[k + i - 8]);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] = fmaxf(acc[i], y[56 + i]);
       const float mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
                                 fmaxf(acc[6], acc[7]));
       const float mx = mraw * sc;  // sc > 0: max of the scaled scores
@@ -315,36 +341,39 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
       const float m_use = grow ? m_new : m_run;
       const float alpha = grow ? fast_exp2(m_run - m_use) : 1.f;
       const float nref = m_use == -INFINITY ? 0.f : -m_use;
-      // p = 2^(s * sc - m): packed FMAs, then MUFU ex2; 8 independent sum chains
+      // p = 2^(s * sc - m) over this thread's half: packed FMAs, MUFU ex2,
+      // 8 independent partial sums
       float sacc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int n = 0; n < 128; n += 2) {
+      for (int n = 0; n < 64; n += 2) {
         ffma2(x[n], x[n + 1], x[n], x[n + 1], sc, sc, nref, nref);
         x[n] = fast_exp2(x[n]);
         x[n + 1] = fast_exp2(x[n + 1]);
       }
 #pragma unroll
-      for (int n = 0; n < 128; n += 16)
+      for (int n = 0; n < 64; n += 16)
 #pragma unroll
-        for (int i = 0; i < 8; i += 2)
-          fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i], x[n + 2 * i + 1]),
+        for (int i = 0; i < 8; i += 2) {
+          fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i], x[n + 2 * i + 1]);
           fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i + 2], x[n + 2 * i + 3]);
+        }
       const float rsum = ((sacc[0] + sacc[1]) + (sacc[2] + sacc[3])) +
                          ((sacc[4] + sacc[5]) + (sacc[6] + sacc[7]));
       if (j > 0) {
         if (!wait_all(&bars[B_OFULL], (j - 1) & 1)) { ok = false; break; }
         tc_fence_after();
-        // rescale O rows whose reference max moved (with real content)
+        // rescale this half of the O row when the reference max moved (with real content)
         const bool need = grow && m_run > -INFINITY;
         if (__any_sync(0xffffffffu, need)) {
 #pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
+          for (int c = 0; c < D / 64; ++c) {
             float o[32];
-            tmem_ld32(tmem + lane_base + C::kColO + 32 * c, o);
+            const uint32_t oc = tmem + lane_base + C::kColO + half * (D / 2) + 32 * c;
+            tmem_ld32(oc, o);
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 32; ++i) o[i] *= alpha;
-            tmem_st32(tmem + lane_base + C::kColO + 32 * c, o);
+            tmem_st32(oc, o);
           }
           tmem_wait_st();
         }
@@ -352,53 +381,64 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
       l_run = l_run * alpha + rsum;
       m_run = m_use;
       if (t.nvalid < 128) {
-        // keys past the range: zero their V rows (stale data may not be finite)
+        // keys past the range: zero their V rows (stale data may not be finite);
+        // each half zeroes its own 64-dim chunk (or its half of the only chunk)
         if (!wait_all(&bars[B_VFULL + s], (j >> 1) & 1)) { ok = false; break; }
         if (row >= t.nvalid) {
           uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
-#pragma unroll
-          for (int c = 0; c < C::NCH; ++c)
+          if (C::NCH == 2) {
 #pragma unroll
             for (int u = 0; u < 8; ++u)
-              *reinterpret_cast<uint4*>(vst + c * C::kChunk + swz128(row, u)) =
+              *reinterpret_cast<uint4*>(vst + half * C::kChunk + swz128(row, u)) =
                   make_uint4(0, 0, 0, 0);
+          } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+              *reinterpret_cast<uint4*>(vst + swz128(row, 4 * half + u)) = make_uint4(0, 0, 0, 0);
+          }
         }
       }
+      // this half of the P row: keys own .. own+63 = P chunk `half`
 #pragma unroll
-      for (int u = 0; u < 16; ++u) {
+      for (int u = 0; u < 8; ++u) {
         uint4 v;
         v.x = pack_bf16(x[8 * u + 0], x[8 * u + 1]);
         v.y = pack_bf16(x[8 * u + 2], x[8 * u + 3]);
         v.z = pack_bf16(x[8 * u + 4], x[8 * u + 5]);
         v.w = pack_bf16(x[8 * u + 6], x[8 * u + 7]);
-        *reinterpret_cast<uint4*>(ps + (u >> 3) * C::kChunk + swz128(row, u & 7)) = v;
+        *reinterpret_cast<uint4*>(ps + half * C::kChunk + swz128(row, u)) = v;
       }
       fence_proxy_async();
       tc_fence_before();
       mbar_arrive(&bars[B_PFULL]);
     }
+    // combine the two halves' partial row sums
+    lpart[half * 128 + row] = l_run;
+    asm volatile("bar.sync 2, 256;" ::: "memory");
+    const float l_tot = lpart[row] + lpart[128 + row];
     if (ok && ntiles > 0) {
       ok = wait_all(&bars[B_OFULL], (ntiles - 1) & 1);
       if (ok) {
         tc_fence_after();
-        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+        const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
+        for (int c = 0; c < D / 64; ++c) {
           float o[32];
-          tmem_ld32(tmem + lane_base + C::kColO + 32 * c, o);
+          const int col = half * (D / 2) + 32 * c;
+          tmem_ld32(tmem + lane_base + C::kColO + col, o);
           tmem_wait_ld();
           if (row_valid) {
             if (item.out_mode == 0) {
               const int64_t slot =
                   dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
-              float4* dst = reinterpret_cast<float4*>(p.part_o + slot * D + 32 * c);
+              float4* dst = reinterpret_cast<float4*>(p.part_o + slot * D + col);
 #pragma unroll
               for (int i = 0; i < 8; ++i)
                 dst[i] = make_float4(o[4 * i] * inv, o[4 * i + 1] * inv, o[4 * i + 2] * inv,
                                      o[4 * i + 3] * inv);
             } else {
               uint4* dst = reinterpret_cast<uint4*>(
-                  p.out + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D + 32 * c);
+                  p.out + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D + col);
 #pragma unroll
               for (int i = 0; i < 4; ++i) {
                 uint4 v;
@@ -411,8 +451,8 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
             }
           }
         }
-        if (row_valid) {
-          const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : -INFINITY;
+        if (row_valid && half == 0) {
+          const float lse = l_tot > 0.f ? (m_run + __log2f(l_tot)) * kLn2 : -INFINITY;
           if (item.out_mode == 0) {
             const int64_t slot = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
             p.part_lse[slot] = lse;
@@ -439,7 +479,7 @@ __global__ void __launch_bounds__(192, 1) dense_kernel(const __grid_constant__ D
 
 template <int D, int G>
 cudaError_t launch_dense_t(const DenseParams& p, int n_items, cudaStream_t stream) {
-  dense_kernel<D, G><<<n_items, 192, DenseCfg<D>::kSmem, stream>>>(p);
+  dense_kernel<D, G><<<n_items, kThreads, DenseCfg<D>::kSmem, stream>>>(p);
   return cudaGetLastError();
 }
 
