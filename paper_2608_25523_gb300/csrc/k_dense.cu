@@ -13,11 +13,13 @@
 // One CTA = one work item (a 128-row Q tile against up to two key segments).
 //   warp 0      TMA producer: K and V tiles (8 pages x 64-dim boxes, 128B
 //               swizzle) into a 2-stage ring, page ids fetched a tile ahead
+//               with independent loads
 //   warp 1      TMEM owner; one lane issues tcgen05.mma:
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
 //                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
-//               QK of tile j+1 is issued before PV of tile j, so the
-//               softmax of j+1 overlaps the tensor work of j
+//               issuing whichever is ready first (QK may run up to two
+//               tiles ahead of PV), so the softmax of tile j+1 overlaps the
+//               tensor work of tile j
 //   warps 2..9  softmax, two warps per TMEM lane quarter: warp 2+q+4h owns
 //               rows 32q..32q+31 and key half h (64 keys).  Both warps of a
 //               pair compute the full-row max (so their running max agrees
@@ -168,15 +170,18 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       auto fetch = [&](int j, int* z) {  // page ids of tile j (0 when past the range)
         const TileInfo t = tile_at(item, j);
         const int npg = (t.nvalid + kPage - 1) / kPage;
+        int32_t pid[8];
+        // independent read-only loads first (one round trip), validation after
+#pragma unroll
+        for (int i = 0; i < 8; ++i) pid[i] = i < npg ? __ldg(p.pages + t.page_off + i) : 0;
+        bool bad = false;
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          int64_t pid = i < npg ? p.pages[t.page_off + i] : 0;
-          if (pid < 0 || pid >= p.num_pages) {
-            atomicOr(p.status, kStatusBadPage);
-            pid = 0;
-          }
-          z[i] = static_cast<int>(pid * p.hkv + item.kv_head);
+          const bool b = pid[i] < 0 || pid[i] >= p.num_pages;
+          bad |= b;
+          z[i] = (b ? 0 : pid[i]) * p.hkv + item.kv_head;
         }
+        if (bad) atomicOr(p.status, kStatusBadPage);
       };
       int znext[8];
       if (ntiles > 0) fetch(0, znext);
@@ -235,31 +240,8 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       const uint32_t pbase = smem_u32(smem + C::kOffP);
       const uint32_t kbase0 = smem_u32(smem + C::kOffK);
       const uint32_t vbase0 = smem_u32(smem + C::kOffV);
-      bool ok = true;
-      auto issue_pv = [&](int i) -> bool {
-        const int s = i & 1;
-        if (!mbar_wait(&bars[B_PFULL], i & 1, abort_flag)) return false;
-        if (!mbar_wait(&bars[B_VFULL + s], (i >> 1) & 1, abort_flag)) return false;
-        tc_fence_after();
-        const uint32_t vb = vbase0 + s * C::kKVBytes;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t a = umma_sdesc(pbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
-          const uint64_t b = umma_sdesc(vb + kk * 2048, C::kChunk, 1024);
-          umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(&bars[B_OFULL]);
-        umma_commit(&bars[B_VEMPTY + s]);
-        return true;
-      };
-      for (int j = 0; j < ntiles && ok; ++j) {
+      auto issue_qk = [&](int j) {
         const int s = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        if (!mbar_wait(&bars[B_KFULL + s], ph, abort_flag) ||
-            !mbar_wait(&bars[B_SFREE + s], ph ^ 1u, abort_flag)) {
-          ok = false;
-          break;
-        }
         tc_fence_after();
         const uint32_t kb = kbase0 + s * C::kKVBytes;
         const uint32_t scol = s ? C::kColS1 : C::kColS0;
@@ -271,9 +253,50 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         }
         umma_commit(&bars[B_SFULL + s]);
         umma_commit(&bars[B_KEMPTY + s]);
-        if (j > 0) ok = issue_pv(j - 1);
+      };
+      auto issue_pv = [&](int i) {
+        const int s = i & 1;
+        tc_fence_after();
+        const uint32_t vb = vbase0 + s * C::kKVBytes;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t a = umma_sdesc(pbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
+          const uint64_t b = umma_sdesc(vb + kk * 2048, C::kChunk, 1024);
+          umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&bars[B_OFULL]);
+        umma_commit(&bars[B_VEMPTY + s]);
+      };
+      // Issue whichever is ready first: QK of the next tile (K landed, its S
+      // buffer released by the softmax two tiles back) or PV of the oldest
+      // tile whose P is written (and V landed).  PVs stay in tile order.
+      bool ok = true;
+      int nq = 0, np = 0;
+      unsigned long long t_last = global_ns();
+      while (ok && np < ntiles) {
+        bool progressed = false;
+        if (nq < ntiles && nq <= np + 2) {
+          const int s = nq & 1;
+          const uint32_t ph = (nq >> 1) & 1;
+          if (mbar_try_wait(&bars[B_KFULL + s], ph) && mbar_try_wait(&bars[B_SFREE + s], ph ^ 1u)) {
+            issue_qk(nq++);
+            progressed = true;
+          }
+        }
+        if (np < nq) {
+          const int s = np & 1;
+          if (mbar_try_wait(&bars[B_PFULL], np & 1) &&
+              mbar_try_wait(&bars[B_VFULL + s], (np >> 1) & 1)) {
+            issue_pv(np++);
+            progressed = true;
+          }
+        }
+        if (progressed) {
+          t_last = global_ns();
+        } else if (*abort_flag || global_ns() - t_last > kWaitLimitNs) {
+          ok = false;
+        }
       }
-      if (ok && ntiles > 0) ok = issue_pv(ntiles - 1);
       if (!ok) {
         *abort_flag = 1;
         atomicOr(p.status, kStatusDenseTimeout);
