@@ -12,8 +12,8 @@
 //
 // One CTA = one work item (a 128-row Q tile against up to two key segments).
 //   warp 0      TMA producer: K and V tiles (8 pages x 64-dim boxes, 128B
-//               swizzle) into a 2-stage ring, page ids fetched a tile ahead
-//               with independent loads
+//               swizzle) into a 2-stage ring; lane i loads page i's id a
+//               tile ahead and issues that page's boxes
 //   warp 1      TMEM owner; one lane issues tcgen05.mma:
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
 //                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
@@ -164,71 +164,63 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
-      bool pok = true;
-      auto fetch = [&](int j, int* z) {  // page ids of tile j (0 when past the range)
-        const TileInfo t = tile_at(item, j);
-        const int npg = (t.nvalid + kPage - 1) / kPage;
-        int32_t pid[8];
-        // independent read-only loads first (one round trip), validation after
+    // Lane i (< 8) owns page i of every tile: it loads that page id one tile
+    // ahead and issues the page's TMA boxes, so a tile's boxes go out from 8
+    // lanes at once.  Lane 0 posts the expected byte count first.
+    int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
+    bool pok = true;
+    auto page_z = [&](int j) {  // this lane's (page, kv head) box row of tile j
+      const TileInfo t = tile_at(item, j);
+      const int npg = (t.nvalid + kPage - 1) / kPage;
+      const int32_t pid = lane < npg ? __ldg(p.pages + t.page_off + lane) : 0;
+      const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
+      if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
+      return (bad ? 0 : pid) * p.hkv + item.kv_head;
+    };
+    auto wait_all = [&](uint64_t* bar, uint32_t parity) {
+      return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
+    };
+    int znext = ntiles > 0 ? page_z(0) : 0;
+    for (int j = 0; j < ntiles; ++j) {
+      const TileInfo t = tile_at(item, j);
+      const int s = j & 1;
+      const uint32_t ph = (j >> 1) & 1;
+      const int npg = (t.nvalid + kPage - 1) / kPage;
+      const uint32_t bytes = static_cast<uint32_t>(npg * C::NCH * 2048);
+      const int z = znext;
+      if (j + 1 < ntiles) znext = page_z(j + 1);
+      if (!wait_all(&bars[B_KEMPTY + s], ph ^ 1u)) { pok = false; break; }
+      if (lane == 0) mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
+      __syncwarp();
+      if (lane < npg) {
+        uint8_t* kst = smem + C::kOffK + s * C::kKVBytes + lane * 2048;
 #pragma unroll
-        for (int i = 0; i < 8; ++i) pid[i] = i < npg ? __ldg(p.pages + t.page_off + i) : 0;
-        bool bad = false;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const bool b = pid[i] < 0 || pid[i] >= p.num_pages;
-          bad |= b;
-          z[i] = (b ? 0 : pid[i]) * p.hkv + item.kv_head;
-        }
-        if (bad) atomicOr(p.status, kStatusBadPage);
-      };
-      int znext[8];
-      if (ntiles > 0) fetch(0, znext);
-      for (int j = 0; j < ntiles; ++j) {
-        const TileInfo t = tile_at(item, j);
-        const int s = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        const int npg = (t.nvalid + kPage - 1) / kPage;
-        const uint32_t bytes = static_cast<uint32_t>(npg * C::NCH * 2048);
-        int z[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) z[i] = znext[i];
-        if (j + 1 < ntiles) fetch(j + 1, znext);
-        if (!mbar_wait(&bars[B_KEMPTY + s], ph ^ 1u, abort_flag)) { pok = false; break; }
-        mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
-        uint8_t* kst = smem + C::kOffK + s * C::kKVBytes;
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          if (i < npg)
-#pragma unroll
-            for (int c = 0; c < C::NCH; ++c)
-              tma_load_3d(kst + c * C::kChunk + i * 2048, &p.tmap_k, &bars[B_KFULL + s], c * 64,
-                          0, z[i]);
-        kph_last[s] = static_cast<int>(ph);
-        if (!mbar_wait(&bars[B_VEMPTY + s], ph ^ 1u, abort_flag)) { pok = false; break; }
-        mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
-        uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          if (i < npg)
-#pragma unroll
-            for (int c = 0; c < C::NCH; ++c)
-              tma_load_3d(vst + c * C::kChunk + i * 2048, &p.tmap_v, &bars[B_VFULL + s], c * 64,
-                          0, z[i]);
-        vph_last[s] = static_cast<int>(ph);
+        for (int c = 0; c < C::NCH; ++c)
+          tma_load_3d(kst + c * C::kChunk, &p.tmap_k, &bars[B_KFULL + s], c * 64, 0, z);
       }
-      if (!pok) {
-        *abort_flag = 1;
-        atomicOr(p.status, kStatusDenseTimeout);
+      kph_last[s] = static_cast<int>(ph);
+      if (!wait_all(&bars[B_VEMPTY + s], ph ^ 1u)) { pok = false; break; }
+      if (lane == 0) mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
+      __syncwarp();
+      if (lane < npg) {
+        uint8_t* vst = smem + C::kOffV + s * C::kKVBytes + lane * 2048;
+#pragma unroll
+        for (int c = 0; c < C::NCH; ++c)
+          tma_load_3d(vst + c * C::kChunk, &p.tmap_v, &bars[B_VFULL + s], c * 64, 0, z);
       }
-      if (*abort_flag) {
-        // let every issued copy land before the CTA's shared memory goes away
-        volatile int never = 0;
-        for (int s = 0; s < 2; ++s) {
-          if (kph_last[s] >= 0) (void)mbar_wait(&bars[B_KFULL + s], kph_last[s], &never);
-          if (vph_last[s] >= 0) (void)mbar_wait(&bars[B_VFULL + s], vph_last[s], &never);
-        }
+      vph_last[s] = static_cast<int>(ph);
+    }
+    if (!pok && lane == 0) {
+      *abort_flag = 1;
+      atomicOr(p.status, kStatusDenseTimeout);
+    }
+    __syncwarp();
+    if (*abort_flag && lane == 0) {
+      // let every issued copy land before the CTA's shared memory goes away
+      volatile int never = 0;
+      for (int s = 0; s < 2; ++s) {
+        if (kph_last[s] >= 0) (void)mbar_wait(&bars[B_KFULL + s], kph_last[s], &never);
+        if (vph_last[s] >= 0) (void)mbar_wait(&bars[B_VFULL + s], vph_last[s], &never);
       }
     }
   } else if (warp == 1) {
