@@ -471,7 +471,9 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
   if ((e = tpa::init_kernels()) != cudaSuccess)
     return cleanup(fail(TPA_ERR_CUDA, "kernel attributes: %s", cudaGetErrorString(e)));
 
-  // TMA descriptors: 3-D view (d, 16 slots, pages*hkv) of each pool, 64x16 boxes
+  // TMA descriptors: a 5-D view of each pool in which one box is one page of
+  // one kv head, (64 dims, 8 slots, d/64 chunks, 2 slot halves, page*hkv), so
+  // it lands as [slot half][chunk][8 slots][128 B] with 128-byte swizzle
   void* fn = nullptr;
   cudaDriverEntryPointQueryResult q;
   if ((e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
@@ -479,14 +481,14 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
       q != cudaDriverEntryPointSuccess || !fn)
     return cleanup(fail(TPA_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable"));
   auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-  const cuuint64_t dims[3] = {static_cast<cuuint64_t>(ctx->d), static_cast<cuuint64_t>(kPage),
-                              static_cast<cuuint64_t>(cfg->num_pages * ctx->hkv)};
-  const cuuint64_t strides[2] = {static_cast<cuuint64_t>(ctx->d) * 2,
-                                 static_cast<cuuint64_t>(kPage) * ctx->d * 2};
-  const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(kPage), 1};
-  const cuuint32_t estr[3] = {1, 1, 1};
+  const cuuint64_t row = static_cast<cuuint64_t>(ctx->d) * 2;  // bytes of one slot's d-row
+  const cuuint64_t nch = static_cast<cuuint64_t>(ctx->d / 64);
+  const cuuint64_t dims[5] = {64, 8, nch, 2, static_cast<cuuint64_t>(cfg->num_pages * ctx->hkv)};
+  const cuuint64_t strides[4] = {row, 128, 8 * row, static_cast<cuuint64_t>(kPage) * row};
+  const cuuint32_t box[5] = {64, 8, static_cast<cuuint32_t>(nch), 2, 1};
+  const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
   for (int w = 0; w < 2; ++w) {
-    CUresult r = encode(w ? &ctx->tmap_v : &ctx->tmap_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+    CUresult r = encode(w ? &ctx->tmap_v : &ctx->tmap_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5,
                         w ? cfg->v_pool : cfg->k_pool, dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);

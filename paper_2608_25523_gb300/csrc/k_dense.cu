@@ -11,9 +11,9 @@
 // request's own suffix.
 //
 // One CTA = one work item (a 128-row Q tile against up to two key segments).
-//   warp 0      TMA producer: K and V tiles (8 pages x 64-dim boxes, 128B
-//               swizzle) into a 2-stage ring; lane i loads page i's id a
-//               tile ahead and issues that page's boxes
+//   warp 0      TMA producer: K and V tiles (8 pages, one 128B-swizzled box
+//               per page and operand) into a 2-stage ring; lane i loads page
+//               i's id a tile ahead and issues that page's boxes
 //   warp 1      TMEM owner; one lane issues tcgen05.mma:
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
 //                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
@@ -55,7 +55,9 @@ struct DenseCfg {
   static constexpr int kChunk = 128 * 128;         // one chunk of a 128-row/128-key tile
   static constexpr int kQBytes = NCH * kChunk;     // Q   [chunk][row][128 B]
   static constexpr int kPBytes = 2 * kChunk;       // P   [key chunk][row][128 B]
-  static constexpr int kKVBytes = NCH * kChunk;    // K,V [chunk][key][128 B]
+  static constexpr int kKVBytes = NCH * kChunk;    // K,V 8 pages, see kv_off
+  static constexpr int kPageBytes = NCH * 2048;    // one page of one kv head
+  static constexpr int kGroup = NCH * 1024;        // stride of 8-key groups
   static constexpr int kStages = 2;
   static constexpr int kOffQ = 0;
   static constexpr int kOffP = kOffQ + kQBytes;
@@ -192,22 +194,16 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       if (!wait_all(&bars[B_KEMPTY + s], ph ^ 1u)) { pok = false; break; }
       if (lane == 0) mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
       __syncwarp();
-      if (lane < npg) {
-        uint8_t* kst = smem + C::kOffK + s * C::kKVBytes + lane * 2048;
-#pragma unroll
-        for (int c = 0; c < C::NCH; ++c)
-          tma_load_3d(kst + c * C::kChunk, &p.tmap_k, &bars[B_KFULL + s], c * 64, 0, z);
-      }
+      if (lane < npg)
+        tma_load_5d(smem + C::kOffK + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_k,
+                    &bars[B_KFULL + s], 0, 0, 0, 0, z);
       kph_last[s] = static_cast<int>(ph);
       if (!wait_all(&bars[B_VEMPTY + s], ph ^ 1u)) { pok = false; break; }
       if (lane == 0) mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
       __syncwarp();
-      if (lane < npg) {
-        uint8_t* vst = smem + C::kOffV + s * C::kKVBytes + lane * 2048;
-#pragma unroll
-        for (int c = 0; c < C::NCH; ++c)
-          tma_load_3d(vst + c * C::kChunk, &p.tmap_v, &bars[B_VFULL + s], c * 64, 0, z);
-      }
+      if (lane < npg)
+        tma_load_5d(smem + C::kOffV + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_v,
+                    &bars[B_VFULL + s], 0, 0, 0, 0, z);
       vph_last[s] = static_cast<int>(ph);
     }
     if (!pok && lane == 0) {
@@ -240,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint64_t a = umma_sdesc(qbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
-          const uint64_t b = umma_sdesc(kb + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
+          const uint64_t b = umma_sdesc(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, C::kGroup);
           umma_bf16_ss(tmem + scol, a, b, idesc_qk, kk > 0 ? 1u : 0u);
         }
         umma_commit(&bars[B_SFULL + s]);
@@ -253,7 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint64_t a = umma_sdesc(pbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
-          const uint64_t b = umma_sdesc(vb + kk * 2048, C::kChunk, 1024);
+          const uint64_t b = umma_sdesc(vb + kk * C::kPageBytes, 1024, C::kGroup);
           umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
         }
         umma_commit(&bars[B_OFULL]);
@@ -404,12 +400,13 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           if (C::NCH == 2) {
 #pragma unroll
             for (int u = 0; u < 8; ++u)
-              *reinterpret_cast<uint4*>(vst + half * C::kChunk + swz128(row, u)) =
+              *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(row, 8 * half + u)) =
                   make_uint4(0, 0, 0, 0);
           } else {
 #pragma unroll
             for (int u = 0; u < 4; ++u)
-              *reinterpret_cast<uint4*>(vst + swz128(row, 4 * half + u)) = make_uint4(0, 0, 0, 0);
+              *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(row, 4 * half + u)) =
+                  make_uint4(0, 0, 0, 0);
           }
         }
       }

@@ -9,8 +9,8 @@
 // the flat cross-check mode.
 //
 // Design (memory-bound: ~4 flop per KV byte at G=4):
-//  * each page of one kv head is two TMA boxes per operand (64 dims x 16
-//    slots, 128-byte swizzle) landing in a per-warp ring of kStages stages,
+//  * each page of one kv head is one TMA box per operand (128-byte swizzle)
+//    landing in a per-warp ring of kStages stages,
 //    so loads run kStages pages ahead of the math;
 //  * S^T tiles use mma.sync m16n8k16 with the G query rows on the M side
 //    (padded to 16) and the 16 keys of the page on N; P*V reuses the S
@@ -109,10 +109,8 @@ __global__ void __launch_bounds__(128) suffix_kernel(const __grid_constant__ Suf
       const int z = static_cast<int>(pid * p.hkv + item.kv_head);
       fence_proxy_async();
       mbar_arrive_expect_tx(&bars[st], 2 * C::kPageBytes);
-#pragma unroll
-      for (int c = 0; c < C::NCH; ++c) tma_load_3d(kst + c * 2048, &p.tmap_k, &bars[st], c * 64, 0, z);
-#pragma unroll
-      for (int c = 0; c < C::NCH; ++c) tma_load_3d(vst + c * 2048, &p.tmap_v, &bars[st], c * 64, 0, z);
+      tma_load_5d(kst, &p.tmap_k, &bars[st], 0, 0, 0, 0, z);
+      tma_load_5d(vst, &p.tmap_v, &bars[st], 0, 0, 0, 0, z);
       ++issued;
     };
 
@@ -144,8 +142,7 @@ __global__ void __launch_bounds__(128) suffix_kernel(const __grid_constant__ Suf
         for (int u = lane; u < nunits; u += 32) {
           const int key = valid + u / (C::NCH * 8);
           const int cu = u % (C::NCH * 8);
-          *reinterpret_cast<uint4*>(vst + (cu >> 3) * 2048 + swz128(key, cu & 7)) =
-              make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(key, cu)) = make_uint4(0, 0, 0, 0);
         }
         __syncwarp();
       }
@@ -161,7 +158,7 @@ __global__ void __launch_bounds__(128) suffix_kernel(const __grid_constant__ Suf
         for (int kk = 0; kk < D / 16; ++kk) {
           const int unit = 2 * kk + usel;
           uint32_t b0, b1, b2, b3;
-          ldmatrix_x4(kbase + (unit >> 3) * 2048 + swz128(key, unit & 7), b0, b1, b2, b3);
+          ldmatrix_x4(kbase + kv_off<C::NCH>(key, unit), b0, b1, b2, b3);
           mma_bf16_16816(s0, qa[kk][0], 0u, qa[kk][1], 0u, b0, b1);
           mma_bf16_16816(s1, qa[kk][0], 0u, qa[kk][1], 0u, b2, b3);
         }
@@ -197,7 +194,7 @@ __global__ void __launch_bounds__(128) suffix_kernel(const __grid_constant__ Suf
         for (int np = 0; np < D / 16; ++np) {
           const int unit = 2 * np + (mat >> 1);
           uint32_t b0, b1, b2, b3;
-          ldmatrix_x4_trans(vbase + (unit >> 3) * 2048 + swz128(key, unit & 7), b0, b1, b2, b3);
+          ldmatrix_x4_trans(vbase + kv_off<C::NCH>(key, unit), b0, b1, b2, b3);
           mma_bf16_16816(o[2 * np], pa0, 0u, pa2, 0u, b0, b1);
           mma_bf16_16816(o[2 * np + 1], pa0, 0u, pa2, 0u, b2, b3);
         }

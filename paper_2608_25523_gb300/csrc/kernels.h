@@ -31,7 +31,7 @@ cudaError_t launch_page_copy(const int32_t* pages, int len, int to_pages, const 
                              const PoolGeom& pool, uint32_t* status, cudaStream_t stream);
 
 struct DenseParams {
-  CUtensorMap tmap_k;  // 3-D view of the K pool: (d, 16 slots, pages*hkv), 64x16 boxes
+  CUtensorMap tmap_k;  // 5-D view of the K pool: one box = one page of one kv head
   CUtensorMap tmap_v;
   const __nv_bfloat16* q;
   __nv_bfloat16* out;

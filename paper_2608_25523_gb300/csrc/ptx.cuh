@@ -79,6 +79,17 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, uint64_
       : "memory");
 }
 
+// 5-D tiled tensor load into shared memory, completion counted on `bar`.
+__device__ __forceinline__ void tma_load_5d(void* dst, const void* tmap, uint64_t* bar, int c0,
+                                            int c1, int c2, int c3, int c4) {
+  asm volatile(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4),
+      "r"(smem_u32(bar))
+      : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
 }
@@ -258,6 +269,16 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 // 128-byte swizzle used by TMA and tcgen05 (1024-byte aligned atoms).
 __device__ __forceinline__ uint32_t swz128(uint32_t row, uint32_t u) {
   return row * 128u + ((u ^ (row & 7u)) << 4);
+}
+
+// Shared-memory image of KV pages as the pool's TMA view lands them: one
+// page of one kv head is [slot half (2)][64-dim chunk (NCH)][8 slots][128 B],
+// so consecutive 8-key groups are NCH*1024 bytes apart across page
+// boundaries too.  Byte offset of key `n` (counted from the first page),
+// 16-byte unit `u` of its d-row (0 .. 8*NCH-1).
+template <int NCH>
+__device__ __forceinline__ uint32_t kv_off(uint32_t n, uint32_t u) {
+  return (n >> 3) * (NCH * 1024u) + (u >> 3) * 1024u + swz128(n & 7u, u & 7u);
 }
 
 }  // namespace tpa
