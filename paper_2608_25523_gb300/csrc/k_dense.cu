@@ -13,7 +13,7 @@
 // One CTA = one work item (a 128-row Q tile against up to two key segments).
 //   warp 0      TMA producer: K and V tiles (8 pages, one 128B-swizzled box
 //               per page and operand) into a 2-stage ring; lane i loads page
-//               i's id a tile ahead and issues that page's boxes
+//               i's id two tiles ahead and issues that page's boxes
 //   warp 1      TMEM owner; one lane issues tcgen05.mma:
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
 //                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
@@ -166,31 +166,33 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    // Lane i (< 8) owns page i of every tile: it loads that page id one tile
+    // Lane i (< 8) owns page i of every tile: it loads that page id two tiles
     // ahead and issues the page's TMA boxes, so a tile's boxes go out from 8
     // lanes at once.  Lane 0 posts the expected byte count first.
     int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
     bool pok = true;
-    auto page_z = [&](int j) {  // this lane's (page, kv head) box row of tile j
+    // this lane's page id of tile j (raw; validated when used, two tiles later)
+    auto page_id = [&](int j) -> int32_t {
+      if (j >= ntiles) return 0;
       const TileInfo t = tile_at(item, j);
-      const int npg = (t.nvalid + kPage - 1) / kPage;
-      const int32_t pid = lane < npg ? __ldg(p.pages + t.page_off + lane) : 0;
-      const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
-      if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
-      return (bad ? 0 : pid) * p.hkv + item.kv_head;
+      return lane < (t.nvalid + kPage - 1) / kPage ? __ldg(p.pages + t.page_off + lane) : 0;
     };
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
       return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
     };
-    int znext = ntiles > 0 ? page_z(0) : 0;
+    int32_t pid0 = page_id(0), pid1 = page_id(1);
     for (int j = 0; j < ntiles; ++j) {
       const TileInfo t = tile_at(item, j);
       const int s = j & 1;
       const uint32_t ph = (j >> 1) & 1;
       const int npg = (t.nvalid + kPage - 1) / kPage;
       const uint32_t bytes = static_cast<uint32_t>(npg * C::NCH * 2048);
-      const int z = znext;
-      if (j + 1 < ntiles) znext = page_z(j + 1);
+      const int32_t pid = pid0;
+      pid0 = pid1;
+      pid1 = page_id(j + 2);
+      const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
+      if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
+      const int z = (bad ? 0 : pid) * p.hkv + item.kv_head;
       if (!wait_all(&bars[B_KEMPTY + s], ph ^ 1u)) { pok = false; break; }
       if (lane == 0) mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
       __syncwarp();
@@ -266,15 +268,14 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         if (nq < ntiles && nq <= np + 2) {
           const int s = nq & 1;
           const uint32_t ph = (nq >> 1) & 1;
-          if (mbar_try_wait(&bars[B_KFULL + s], ph) && mbar_try_wait(&bars[B_SFREE + s], ph ^ 1u)) {
+          if (mbar_test(&bars[B_KFULL + s], ph) && mbar_test(&bars[B_SFREE + s], ph ^ 1u)) {
             issue_qk(nq++);
             progressed = true;
           }
         }
         if (np < nq) {
           const int s = np & 1;
-          if (mbar_try_wait(&bars[B_PFULL], np & 1) &&
-              mbar_try_wait(&bars[B_VFULL + s], (np >> 1) & 1)) {
+          if (mbar_test(&bars[B_PFULL], np & 1) && mbar_test(&bars[B_VFULL + s], (np >> 1) & 1)) {
             issue_pv(np++);
             progressed = true;
           }
