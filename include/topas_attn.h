@@ -217,12 +217,14 @@ enum {
 TPA_API int tpa_query(tpa_ctx* ctx, int32_t what, int32_t id, int64_t* value);
 
 enum {
-  TPA_OPT_DECODE_MODE = 0,      /* 0: cascade (default); 1: flat -- every key, prefix included,
-                                   through the split-KV kernel (a cross-check path) */
-  TPA_OPT_PREFIX_SPLITS = 1,    /* decode: key splits per stacked prefix tile; 0 = automatic */
-  TPA_OPT_SUFFIX_SPLIT_KEYS = 2,/* split-KV chunk in keys (multiple of 16); 0 = automatic */
-  TPA_OPT_CONCURRENT = 3,       /* 1 (default): prefix and suffix kernels overlap on a forked
-                                   stream; 0: one after the other on the caller's stream */
+  TPA_OPT_DECODE_MODE = 0,      /* 0: cascade (default): one persistent tensor-core launch
+                                   over stacked prefix tiles and per-request suffixes, with the
+                                   KV append and the LSE merge inside; 1: flat cross-check --
+                                   KV append, every key (prefix included) through the split-KV
+                                   kernel, then a separate merge */
+  TPA_OPT_PREFIX_SPLITS = 1,    /* cascade: key splits per stacked prefix tile; 0 = automatic */
+  TPA_OPT_SUFFIX_SPLIT_KEYS = 2,/* keys per suffix work item (cascade: rounded up to 128;
+                                   flat: multiple of 16); 0 = automatic */
   TPA_OPT_KERNEL_TIMING = 4     /* 1: bracket every kernel with CUDA events (tpa_kernel_times) */
 };
 TPA_API int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value);

@@ -88,11 +88,12 @@ struct Slot {
 
 // Sizes of one plan: number of records per section.
 struct PlanSizes {
-  int64_t pages = 0, append = 0, dense_tok = 0, dense = 0, suffix = 0, merge = 0;
+  int64_t pages = 0, append = 0, dense_tok = 0, dense = 0, suffix = 0, merge = 0, counters = 0;
 };
 
 struct PlanLayout {
-  size_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, total;
+  size_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, off_counters,
+      total;
 };
 
 PlanLayout layout_of(const PlanSizes& s) {
@@ -110,6 +111,8 @@ PlanLayout layout_of(const PlanSizes& s) {
   o = align_up(o + s.suffix * sizeof(SuffixItem), 64);
   l.off_merge = o;
   o = align_up(o + s.merge * sizeof(MergeTok), 64);
+  l.off_counters = o;
+  o = align_up(o + s.counters * 4, 64);
   l.total = o;
   return l;
 }
@@ -134,8 +137,6 @@ struct tpa_ctx {
   int num_sms = 148;
   CUtensorMap tmap_k{}, tmap_v{};
   PoolGeom pool{};
-  cudaStream_t fork_stream = nullptr;
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   uint32_t* status = nullptr;
   float* part_o = nullptr;
   float* part_lse = nullptr;
@@ -151,7 +152,6 @@ struct tpa_ctx {
   int decode_mode = 0;
   int prefix_splits = 0;
   int suffix_split_keys = 0;
-  int concurrent = 1;
   int64_t last_dense = 0, last_suffix = 0, last_launches = 0;
 
   // per-kernel event timing (TPA_OPT_KERNEL_TIMING)
@@ -201,13 +201,16 @@ PlanSizes plan_capacity(const tpa_config* c) {
   const int64_t R = max_batch_requests(c);
   const int64_t A = std::min<int64_t>(c->max_agents, R);
   const int64_t S = splits_of(c);
+  const int64_t H = c->num_kv_heads;
   PlanSizes s;
   s.pages = (R + A) * max_pages_of(c);
   s.append = T;
-  s.dense_tok = T;
-  s.dense = c->num_kv_heads * std::max((cdiv(R, tpt) + A) * S, cdiv(T, tpt) + R);
-  s.suffix = R * c->num_kv_heads * S;
+  s.dense_tok = T + R;
+  // decode: stacked prefix tiles + per-token suffix items; prefill: chunk tiles
+  s.dense = H * std::max((cdiv(R, tpt) + A) * S + R * S, cdiv(T, tpt) + R);
+  s.suffix = R * H * S;
   s.merge = R;
+  s.counters = R * H;
   return s;
 }
 
@@ -318,6 +321,7 @@ struct PlanWriter {
   DenseItem* dense;
   SuffixItem* suffix;
   MergeTok* merge;
+  uint32_t* counters;
   PlanWriter(uint8_t* b, const PlanLayout& l) : base(b), lay(l) {
     hdr = reinterpret_cast<PlanHeader*>(b);
     std::memset(hdr, 0, sizeof(PlanHeader));
@@ -327,6 +331,7 @@ struct PlanWriter {
     dense = reinterpret_cast<DenseItem*>(b + l.off_dense);
     suffix = reinterpret_cast<SuffixItem*>(b + l.off_suffix);
     merge = reinterpret_cast<MergeTok*>(b + l.off_merge);
+    counters = reinterpret_cast<uint32_t*>(b + l.off_counters);
   }
 };
 
@@ -515,10 +520,6 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
     if ((e = cudaEventCreateWithFlags(&s.done, cudaEventDisableTiming)) != cudaSuccess)
       return cleanup(fail(TPA_ERR_CUDA, "event: %s", cudaGetErrorString(e)));
   }
-  if ((e = cudaStreamCreateWithFlags(&ctx->fork_stream, cudaStreamNonBlocking)) != cudaSuccess ||
-      (e = cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming)) != cudaSuccess ||
-      (e = cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming)) != cudaSuccess)
-    return cleanup(fail(TPA_ERR_CUDA, "streams: %s", cudaGetErrorString(e)));
   if ((e = cudaMemsetAsync(ctx->status, 0, sizeof(uint32_t), 0)) != cudaSuccess ||
       (e = cudaStreamSynchronize(0)) != cudaSuccess)
     return cleanup(fail(TPA_ERR_CUDA, "status init: %s", cudaGetErrorString(e)));
@@ -539,14 +540,8 @@ int tpa_destroy(tpa_ctx* ctx) {
       }
       if (s.host) cudaFreeHost(s.host);
     }
-    if (ctx->fork_stream) {
-      cudaStreamSynchronize(ctx->fork_stream);
-      cudaStreamDestroy(ctx->fork_stream);
-    }
     resolve_timing(ctx);
     for (cudaEvent_t e : ctx->ev_free) cudaEventDestroy(e);
-    if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
-    if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
   }
   delete ctx;
   return TPA_OK;
@@ -856,7 +851,38 @@ struct AgentGroup {
 
 }  // namespace
 
-// Build and launch a decode step (cascade or flat).
+// Fill the DenseParams common to every dense launch.
+static DenseParams dense_params(tpa_ctx* ctx, const Slot* sl, const PlanLayout& lay, int n_items,
+                                const void* q, void* out, float* lse) {
+  DenseParams dp{};
+  dp.tmap_k = ctx->tmap_k;
+  dp.tmap_v = ctx->tmap_v;
+  dp.q = static_cast<const __nv_bfloat16*>(q);
+  dp.out = static_cast<__nv_bfloat16*>(out);
+  dp.lse = lse;
+  dp.part_o = ctx->part_o;
+  dp.part_lse = ctx->part_lse;
+  dp.items = dev_ptr<DenseItem>(sl, lay.off_dense);
+  dp.toks = dev_ptr<DenseTok>(sl, lay.off_dense_tok);
+  dp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
+  dp.k_pool = static_cast<__nv_bfloat16*>(ctx->cfg.k_pool);
+  dp.v_pool = static_cast<__nv_bfloat16*>(ctx->cfg.v_pool);
+  dp.status = ctx->status;
+  dp.num_pages = ctx->cfg.num_pages;
+  dp.n_items = n_items;
+  dp.hq = ctx->hq;
+  dp.hkv = ctx->hkv;
+  dp.scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(ctx->d));
+  return dp;
+}
+
+// Build and launch a decode step.
+//  cascade (default): one persistent tcgen05 launch.  Work items are the
+//    stacked shared-prefix tiles of each agent (level 1) and, per token and
+//    kv head, its suffix (level 2, which also appends the step's token);
+//    the last partial of each (token, kv head) triggers the in-kernel merge.
+//  flat (cross-check): KV append, the split-KV kernel over every key of
+//    each request (prefix included), and a separate LSE merge.
 int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, const void* k_new,
                const void* v_new, void* out, float* lse, void* stream) {
   if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
@@ -870,6 +896,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
 
   // group tokens by agent (first appearance order)
   std::vector<AgentGroup> groups;
+  std::vector<int32_t> group_of(n);
   {
     std::unordered_map<int32_t, int> gi;
     for (int i = 0; i < n; ++i) {
@@ -881,110 +908,99 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       } else {
         groups[it->second].toks.push_back(i);
       }
+      group_of[i] = gi[a];
     }
   }
+  auto keys_of = [&](int i) -> int64_t { return ctx->reqs[reqs[i]].len + 1; };  // with the new token
+  auto lp_of = [&](int i) -> int64_t { return ctx->agents[ctx->reqs[reqs[i]].agent].len; };
 
-  // split sizes
-  int64_t max_len = 0, sum_keys = 0, max_prefix = 0;
-  for (int i = 0; i < n; ++i) {
-    const Request& r = ctx->reqs[reqs[i]];
-    max_len = std::max<int64_t>(max_len, r.len + 1);
-    sum_keys += r.len + 1;
-    max_prefix = std::max<int64_t>(max_prefix, ctx->agents[r.agent].len);
-    if (flat) sum_keys += ctx->agents[r.agent].len;
-  }
-  int n_units = 0;  // dense (agent, kv head, q tile) units
-  if (!flat)
-    for (auto& g : groups)
-      if (ctx->agents[g.agent].len > 0) n_units += hkv * static_cast<int>(cdiv(g.toks.size(), tpt));
-  int64_t split_keys = ctx->suffix_split_keys;
-  if (split_keys <= 0) {
-    // about two items per resident warp, 64..1024 keys each
-    const int64_t warps = static_cast<int64_t>(ctx->num_sms) * 8;
-    split_keys = cdiv(sum_keys * hkv, 2 * warps);
-    split_keys = std::min<int64_t>(std::max<int64_t>(split_keys, 64), 1024);
-  }
-  split_keys = cdiv(split_keys, kPage) * kPage;
-  for (auto& g : groups) {
-    const int64_t lp = ctx->agents[g.agent].len;
-    if (flat || lp == 0) continue;
-    const int64_t tiles = cdiv(lp, kTileKeys);
-    int64_t ns = ctx->prefix_splits;
-    // one wave: at most as many dense CTAs as SMs
-    if (ns <= 0) ns = std::max<int64_t>(1, ctx->num_sms / std::max(1, n_units));
-    ns = std::min<int64_t>(ns, tiles);
-    g.tiles_per_split = static_cast<int32_t>(cdiv(tiles, ns));
-    g.n_split = static_cast<int32_t>(cdiv(tiles, g.tiles_per_split));
-  }
-  // keep every token's partial count within max_splits
-  {
-    int64_t worst = 0;
-    for (int i = 0; i < n; ++i) {
-      const Request& r = ctx->reqs[reqs[i]];
-      const int64_t lp = ctx->agents[r.agent].len;
-      int64_t nsp = 0;
-      for (auto& g : groups)
-        if (g.agent == r.agent) nsp = g.n_split;
-      const int64_t keys_flat = flat ? lp : 0;
-      worst = std::max(worst, nsp + cdiv(r.len + 1, split_keys) + cdiv(keys_flat, split_keys));
-      if (nsp >= ctx->max_splits) return fail(TPA_ERR_CAPACITY, "prefix splits exceed max_splits");
+  // ---- work decomposition -------------------------------------------------
+  int64_t split_keys = 0;  // suffix (and, flat, prefix) key range per item
+  if (flat) {
+    int64_t sum_keys = 0;
+    for (int i = 0; i < n; ++i) sum_keys += keys_of(i) + lp_of(i);
+    split_keys = ctx->suffix_split_keys;
+    if (split_keys <= 0) {
+      // about two items per resident warp of the split-KV kernel
+      const int64_t warps = static_cast<int64_t>(ctx->num_sms) * 8;
+      split_keys = std::min<int64_t>(std::max<int64_t>(cdiv(sum_keys * hkv, 2 * warps), 64), 1024);
     }
-    while (worst > ctx->max_splits) {
+    split_keys = cdiv(split_keys, kPage) * kPage;
+    for (;;) {
+      int64_t worst = 0;
+      for (int i = 0; i < n; ++i)
+        worst = std::max(worst, cdiv(keys_of(i), split_keys) + cdiv(lp_of(i), split_keys));
+      if (worst <= ctx->max_splits) break;
       split_keys *= 2;
-      worst = 0;
-      for (int i = 0; i < n; ++i) {
-        const Request& r = ctx->reqs[reqs[i]];
-        const int64_t lp = ctx->agents[r.agent].len;
-        int64_t nsp = 0;
-        for (auto& g : groups)
-          if (g.agent == r.agent) nsp = g.n_split;
-        worst = std::max(worst, nsp + cdiv(r.len + 1, split_keys) + cdiv(flat ? lp : 0, split_keys));
-      }
+    }
+  } else {
+    // total key tiles over both levels; aim for items of about one SM's share
+    int64_t tiles = 0;
+    for (auto& g : groups)
+      tiles += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) *
+               cdiv(ctx->agents[g.agent].len, kTileKeys);
+    for (int i = 0; i < n; ++i) tiles += hkv * cdiv(keys_of(i), kTileKeys);
+    const int64_t target = std::max<int64_t>(4, cdiv(tiles, ctx->num_sms));
+    for (auto& g : groups) {
+      const int64_t ptiles = cdiv(ctx->agents[g.agent].len, kTileKeys);
+      if (ptiles == 0) continue;
+      int64_t ns = ctx->prefix_splits > 0 ? ctx->prefix_splits : cdiv(ptiles, target);
+      ns = std::min<int64_t>(std::max<int64_t>(ns, 1), ptiles);
+      g.tiles_per_split = static_cast<int32_t>(cdiv(ptiles, ns));
+      g.n_split = static_cast<int32_t>(cdiv(ptiles, g.tiles_per_split));
+      if (g.n_split >= ctx->max_splits)
+        return fail(TPA_ERR_CAPACITY, "prefix splits exceed max_splits");
+    }
+    split_keys = ctx->suffix_split_keys > 0 ? ctx->suffix_split_keys : target * kTileKeys;
+    split_keys = cdiv(split_keys, kTileKeys) * kTileKeys;
+    for (;;) {
+      int64_t worst = 0;
+      for (int i = 0; i < n; ++i)
+        worst = std::max<int64_t>(worst, groups[group_of[i]].n_split + cdiv(keys_of(i), split_keys));
+      if (worst <= ctx->max_splits) break;
+      split_keys *= 2;
     }
   }
-
-  std::vector<int32_t> ones(n, 1);
-
-  // sizes (suffix page counts after this step's append)
-  PlanSizes sz;
-  sz.append = n;
-  sz.merge = n;
-  sz.dense_tok = n;
-  for (auto& g : groups) sz.pages += ctx->agents[g.agent].pages.size();
-  for (int i = 0; i < n; ++i) sz.pages += cdiv(ctx->reqs[reqs[i]].len + 1, kPage);
-  int64_t n_dense = 0, n_suffix = 0;
-  for (auto& g : groups) n_dense += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) * g.n_split;
-  for (int i = 0; i < n; ++i) {
-    const Request& r = ctx->reqs[reqs[i]];
-    n_suffix += hkv * (cdiv(r.len + 1, split_keys) + (flat ? cdiv(ctx->agents[r.agent].len, split_keys) : 0));
-  }
-  sz.dense = n_dense;
-  sz.suffix = n_suffix;
-  const PlanLayout lay = layout_of(sz);
-  if (lay.total > ctx->plan_cap) return fail(TPA_ERR_CAPACITY, "plan of %zu bytes > %zu", lay.total, ctx->plan_cap);
 
   // partial slots per token
-  std::vector<int32_t> nsp_of(n, 0), slot_base(n), n_slots(n);
-  for (auto& g : groups)
-    for (int32_t i : g.toks) nsp_of[i] = g.n_split;
+  std::vector<int32_t> slot_base(n), n_slots(n);
   int64_t slots = 0;
   for (int i = 0; i < n; ++i) {
-    const Request& r = ctx->reqs[reqs[i]];
-    const int64_t lp = ctx->agents[r.agent].len;
-    n_slots[i] = static_cast<int32_t>(nsp_of[i] + cdiv(r.len + 1, split_keys) + (flat ? cdiv(lp, split_keys) : 0));
+    const int64_t ns = flat ? cdiv(lp_of(i), split_keys) + cdiv(keys_of(i), split_keys)
+                            : groups[group_of[i]].n_split + cdiv(keys_of(i), split_keys);
+    n_slots[i] = static_cast<int32_t>(ns);
     slot_base[i] = static_cast<int32_t>(slots);
-    slots += static_cast<int64_t>(hq) * n_slots[i];
+    slots += static_cast<int64_t>(hq) * ns;
   }
   if (slots > ctx->part_slots) return fail(TPA_ERR_CAPACITY, "partial slots exhausted");
 
+  // plan sizes (suffix page counts after this step's append)
+  PlanSizes sz;
+  for (auto& g : groups) sz.pages += ctx->agents[g.agent].pages.size();
+  for (int i = 0; i < n; ++i) sz.pages += cdiv(keys_of(i), kPage);
+  if (flat) {
+    sz.append = n;
+    sz.merge = n;
+    for (int i = 0; i < n; ++i)
+      sz.suffix += hkv * (cdiv(keys_of(i), split_keys) + cdiv(lp_of(i), split_keys));
+  } else {
+    sz.dense_tok = 2 * n;
+    sz.counters = static_cast<int64_t>(n) * hkv;
+    for (auto& g : groups) sz.dense += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) * g.n_split;
+    for (int i = 0; i < n; ++i) sz.dense += hkv * cdiv(keys_of(i), split_keys);
+  }
+  const PlanLayout lay = layout_of(sz);
+  if (lay.total > ctx->plan_cap)
+    return fail(TPA_ERR_CAPACITY, "plan of %zu bytes > %zu", lay.total, ctx->plan_cap);
+
   // pages for the new tokens (all checks are done: from here on only CUDA errors can fail)
+  std::vector<int32_t> ones(n, 1);
   uint64_t tag = 0;
   if ((rc = reserve_append(ctx, n, reqs, ones.data(), &tag))) return rc;
 
   Slot* sl = acquire_slot(ctx);
   ++ctx->seq;
   PlanWriter w(sl->host, lay);
-  for (int i = 0; i < n; ++i) w.merge[i] = MergeTok{i, slot_base[i], n_slots[i], 0};
 
   // page list: prefixes, then each token's suffix (after the append)
   int32_t np = 0;
@@ -1001,74 +1017,98 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     std::memcpy(w.pages + np, r.pages.data(), r.pages.size() * 4);
     np += static_cast<int32_t>(r.pages.size());
   }
-  write_append_rows(ctx, n, reqs, ones.data(), w.append);
 
-  // level 1: stacked prefix tiles
-  int32_t nt = 0, nd = 0;
-  for (auto& g : groups) {
-    if (g.n_split == 0) continue;
-    const int64_t lp = ctx->agents[g.agent].len;
-    const int nqt = static_cast<int>(cdiv(g.toks.size(), tpt));
-    for (int qt = 0; qt < nqt; ++qt) {
-      const int t0 = qt * tpt;
-      const int t1 = std::min<int>(static_cast<int>(g.toks.size()), t0 + tpt);
-      const int32_t tok_base = nt;
-      for (int t = t0; t < t1; ++t) {
-        const int i = g.toks[t];
-        w.dtok[nt++] = DenseTok{i, 0x7fffffff, slot_base[i], n_slots[i]};
+  int32_t nd = 0, ns = 0, nt = 0;
+  if (flat) {
+    write_append_rows(ctx, n, reqs, ones.data(), w.append);
+    for (int i = 0; i < n; ++i) w.merge[i] = MergeTok{i, slot_base[i], n_slots[i], 0};
+    for (int i = 0; i < n; ++i) {
+      int split = 0;
+      for (int pass = 0; pass < 2; ++pass) {
+        const int64_t len = pass == 0 ? lp_of(i) : keys_of(i);
+        const int32_t base = pass == 0 ? groups[group_of[i]].page_off : suf_off[i];
+        for (int64_t k0 = 0; k0 < len; k0 += split_keys, ++split)
+          for (int h = 0; h < hkv; ++h)
+            w.suffix[ns++] = SuffixItem{i, h, static_cast<int32_t>(base + k0 / kPage),
+                                        static_cast<int32_t>(std::min<int64_t>(split_keys, len - k0)),
+                                        slot_base[i], n_slots[i], split, 0};
       }
-      for (int h = 0; h < hkv; ++h)
-        for (int sp = 0; sp < g.n_split; ++sp) {
+    }
+    std::stable_sort(w.suffix, w.suffix + ns,
+                     [](const SuffixItem& a, const SuffixItem& b) { return a.n_keys > b.n_keys; });
+  } else {
+    std::memset(w.counters, 0, static_cast<size_t>(n) * hkv * 4);
+    // level 1: stacked prefix tiles of each agent
+    for (auto& g : groups) {
+      if (g.n_split == 0) continue;
+      const int64_t lp = ctx->agents[g.agent].len;
+      const int nqt = static_cast<int>(cdiv(g.toks.size(), tpt));
+      for (int qt = 0; qt < nqt; ++qt) {
+        const int t0 = qt * tpt;
+        const int t1 = std::min<int>(static_cast<int>(g.toks.size()), t0 + tpt);
+        const int32_t tok_base = nt;
+        for (int t = t0; t < t1; ++t) {
+          const int i = g.toks[t];
+          w.dtok[nt++] = DenseTok{i, 0x7fffffff, slot_base[i], n_slots[i]};
+        }
+        for (int h = 0; h < hkv; ++h)
+          for (int sp = 0; sp < g.n_split; ++sp) {
+            DenseItem it{};
+            it.tok_base = tok_base;
+            it.n_tok = t1 - t0;
+            it.kv_head = h;
+            it.split = sp;
+            it.out_mode = 0;
+            it.seg_pages[0] = g.page_off;
+            it.seg_k0[0] = static_cast<int32_t>(static_cast<int64_t>(sp) * g.tiles_per_split * kTileKeys);
+            it.seg_k1[0] = static_cast<int32_t>(
+                std::min<int64_t>(lp, static_cast<int64_t>(sp + 1) * g.tiles_per_split * kTileKeys));
+            it.n_tiles = static_cast<int32_t>(cdiv(it.seg_k1[0] - it.seg_k0[0], kTileKeys));
+            it.app_src = -1;
+            w.dense[nd++] = it;
+          }
+      }
+    }
+    // level 2: each token's suffix per kv head; the item holding the last key
+    // appends the step's token first
+    for (int i = 0; i < n; ++i) {
+      const Request& r = ctx->reqs[reqs[i]];
+      const int32_t tok_idx = nt;
+      w.dtok[nt++] = DenseTok{i, 0x7fffffff, slot_base[i], n_slots[i]};
+      const int64_t keys = keys_of(i);
+      const int pos = r.len;  // slot of the new token
+      const int32_t app_dst = r.pages[pos / kPage] * kPage + pos % kPage;
+      int split = groups[group_of[i]].n_split;
+      for (int64_t k0 = 0; k0 < keys; k0 += split_keys, ++split)
+        for (int h = 0; h < hkv; ++h) {
           DenseItem it{};
-          it.tok_base = tok_base;
-          it.n_tok = t1 - t0;
+          it.tok_base = tok_idx;
+          it.n_tok = 1;
           it.kv_head = h;
-          it.split = sp;
+          it.split = split;
           it.out_mode = 0;
-          it.seg_pages[0] = g.page_off;
-          it.seg_k0[0] = static_cast<int32_t>(static_cast<int64_t>(sp) * g.tiles_per_split * kTileKeys);
-          it.seg_k1[0] = static_cast<int32_t>(std::min<int64_t>(lp, static_cast<int64_t>(sp + 1) * g.tiles_per_split * kTileKeys));
-          it.seg_pages[1] = 0;
-          it.seg_k0[1] = it.seg_k1[1] = 0;
+          it.seg_pages[0] = suf_off[i];
+          it.seg_k0[0] = static_cast<int32_t>(k0);
+          it.seg_k1[0] = static_cast<int32_t>(std::min<int64_t>(keys, k0 + split_keys));
           it.n_tiles = static_cast<int32_t>(cdiv(it.seg_k1[0] - it.seg_k0[0], kTileKeys));
+          const bool last = k0 + split_keys >= keys;
+          it.app_src = last ? i : -1;
+          it.app_dst = last ? app_dst : 0;
           w.dense[nd++] = it;
         }
     }
+    std::stable_sort(w.dense, w.dense + nd,
+                     [](const DenseItem& a, const DenseItem& b) { return a.n_tiles > b.n_tiles; });
   }
-  // level 2: split-KV over suffixes (and prefixes in flat mode)
-  int32_t ns = 0;
-  for (int i = 0; i < n; ++i) {
-    const Request& r = ctx->reqs[reqs[i]];
-    const int64_t keys = r.len + 1;
-    const int64_t lp = ctx->agents[r.agent].len;
-    int32_t gpo = 0;
-    for (auto& g : groups)
-      if (g.agent == r.agent) gpo = g.page_off;
-    int split = nsp_of[i];
-    for (int pass = 0; pass < 2; ++pass) {
-      const bool pre = pass == 0;
-      if (pre && !flat) continue;
-      const int64_t len = pre ? lp : keys;
-      const int32_t base = pre ? gpo : suf_off[i];
-      for (int64_t k0 = 0; k0 < len; k0 += split_keys, ++split)
-        for (int h = 0; h < hkv; ++h)
-          w.suffix[ns++] = SuffixItem{i, h, static_cast<int32_t>(base + k0 / kPage),
-                                      static_cast<int32_t>(std::min<int64_t>(split_keys, len - k0)),
-                                      slot_base[i], n_slots[i], split, 0};
-    }
-  }
-  std::stable_sort(w.suffix, w.suffix + ns,
-                   [](const SuffixItem& a, const SuffixItem& b) { return a.n_keys > b.n_keys; });
-  std::stable_sort(w.dense, w.dense + nd,
-                   [](const DenseItem& a, const DenseItem& b) { return a.n_tiles > b.n_tiles; });
 
   PlanHeader* hd = w.hdr;
   hd->n_pages = np;
-  hd->n_append = n;
+  hd->n_append = flat ? n : 0;
   hd->n_dense_tok = nt;
   hd->n_dense = nd;
   hd->n_suffix = ns;
-  hd->n_merge = n;
+  hd->n_merge = flat ? n : 0;
+  hd->n_counters = flat ? 0 : n * hkv;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   chain_begin(ctx, s);
@@ -1078,42 +1118,13 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
 
   int launches = 0;
   if (!ctx->plan_only) {
-    {
-      KernelTimer kt(ctx, K_APPEND, s);
-      CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), n, k_new, v_new, ctx->pool,
-                             ctx->status, s));
-    }
-    ++launches;
     const float scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(ctx->d));
-    cudaStream_t ds = s;
-    const bool fork = ctx->concurrent && nd > 0 && ns > 0;
-    if (fork) {
-      CUDA_TRY(cudaEventRecord(ctx->ev_fork, s));
-      CUDA_TRY(cudaStreamWaitEvent(ctx->fork_stream, ctx->ev_fork, 0));
-      ds = ctx->fork_stream;
-    }
-    if (nd > 0) {
-      DenseParams dp{};
-      dp.tmap_k = ctx->tmap_k;
-      dp.tmap_v = ctx->tmap_v;
-      dp.q = static_cast<const __nv_bfloat16*>(q);
-      dp.out = static_cast<__nv_bfloat16*>(out);
-      dp.lse = lse;
-      dp.part_o = ctx->part_o;
-      dp.part_lse = ctx->part_lse;
-      dp.items = dev_ptr<DenseItem>(sl, lay.off_dense);
-      dp.toks = dev_ptr<DenseTok>(sl, lay.off_dense_tok);
-      dp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
-      dp.status = ctx->status;
-      dp.num_pages = ctx->cfg.num_pages;
-      dp.hq = hq;
-      dp.hkv = hkv;
-      dp.scale_log2 = scale_log2;
-      KernelTimer kt(ctx, K_DENSE, ds);
-      CUDA_TRY(launch_dense(dp, nd, ctx->d, G, ds));
-      ++launches;
-    }
-    if (ns > 0) {
+    if (flat) {
+      {
+        KernelTimer kt(ctx, K_APPEND, s);
+        CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), n, k_new, v_new, ctx->pool,
+                               ctx->status, s));
+      }
       SuffixParams sp{};
       sp.tmap_k = ctx->tmap_k;
       sp.tmap_v = ctx->tmap_v;
@@ -1129,20 +1140,25 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       sp.hq = hq;
       sp.hkv = hkv;
       sp.scale_log2 = scale_log2;
-      KernelTimer kt(ctx, K_SUFFIX, s);
-      CUDA_TRY(launch_suffix(sp, ctx->num_sms, ctx->d, G, s));
-      ++launches;
+      {
+        KernelTimer kt(ctx, K_SUFFIX, s);
+        CUDA_TRY(launch_suffix(sp, ctx->num_sms, ctx->d, G, s));
+      }
+      {
+        KernelTimer kt(ctx, K_MERGE, s);
+        CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
+                              static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, s));
+      }
+      launches = 3;
+    } else {
+      DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
+      dp.k_new = static_cast<const __nv_bfloat16*>(k_new);
+      dp.v_new = static_cast<const __nv_bfloat16*>(v_new);
+      dp.counters = reinterpret_cast<uint32_t*>(sl->dev + lay.off_counters);
+      KernelTimer kt(ctx, K_DENSE, s);
+      CUDA_TRY(launch_dense(dp, ctx->num_sms, ctx->d, G, s));
+      launches = 1;
     }
-    if (fork) {
-      CUDA_TRY(cudaEventRecord(ctx->ev_join, ctx->fork_stream));
-      CUDA_TRY(cudaStreamWaitEvent(s, ctx->ev_join, 0));
-    }
-    {
-      KernelTimer kt(ctx, K_MERGE, s);
-      CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
-                            static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, s));
-    }
-    ++launches;
   }
   for (int i = 0; i < n; ++i) {
     Request& r = ctx->reqs[reqs[i]];
@@ -1246,6 +1262,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
         it.seg_k1[1] = offset[i] + t1;  // keys up to the tile's last position
         it.seg_causal[1] = 1;
         it.n_tiles = static_cast<int32_t>(cdiv(lp, kTileKeys) + cdiv(it.seg_k1[1], kTileKeys));
+        it.app_src = -1;
         w.dense[nd++] = it;
       }
     }
@@ -1270,24 +1287,9 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
       CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
                              v_new, ctx->pool, ctx->status, s));
     }
-    DenseParams dp{};
-    dp.tmap_k = ctx->tmap_k;
-    dp.tmap_v = ctx->tmap_v;
-    dp.q = static_cast<const __nv_bfloat16*>(q);
-    dp.out = static_cast<__nv_bfloat16*>(out);
-    dp.lse = lse;
-    dp.part_o = ctx->part_o;
-    dp.part_lse = ctx->part_lse;
-    dp.items = dev_ptr<DenseItem>(sl, lay.off_dense);
-    dp.toks = dev_ptr<DenseTok>(sl, lay.off_dense_tok);
-    dp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
-    dp.status = ctx->status;
-    dp.num_pages = ctx->cfg.num_pages;
-    dp.hq = hq;
-    dp.hkv = hkv;
-    dp.scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(ctx->d));
+    DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
     KernelTimer kt(ctx, K_DENSE, s);
-    CUDA_TRY(launch_dense(dp, nd, ctx->d, G, s));
+    CUDA_TRY(launch_dense(dp, ctx->num_sms, ctx->d, G, s));
   }
   for (int i = 0; i < n; ++i) {
     Request& r = ctx->reqs[reqs[i]];
@@ -1379,9 +1381,6 @@ int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
         return fail(TPA_ERR_INVALID_ARG, "split keys must be a multiple of 16");
       ctx->suffix_split_keys = static_cast<int>(value);
       return TPA_OK;
-    case TPA_OPT_CONCURRENT:
-      ctx->concurrent = value ? 1 : 0;
-      return TPA_OK;
     case TPA_OPT_KERNEL_TIMING:
       ctx->timing = value ? 1 : 0;
       return TPA_OK;
@@ -1412,7 +1411,6 @@ int tpa_device_status(tpa_ctx* ctx, void* stream, uint32_t* status) {
   if (ctx->plan_only) return TPA_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   CUDA_TRY(cudaStreamSynchronize(s));
-  if (ctx->fork_stream) CUDA_TRY(cudaStreamSynchronize(ctx->fork_stream));
   CUDA_TRY(cudaMemcpy(status, ctx->status, sizeof(uint32_t), cudaMemcpyDeviceToHost));
   CUDA_TRY(cudaMemset(ctx->status, 0, sizeof(uint32_t)));
   if (*status & (kStatusDenseTimeout | kStatusSuffixTimeout))

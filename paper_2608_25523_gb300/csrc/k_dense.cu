@@ -1,36 +1,45 @@
-// Dense tensor-core attention over paged KV (tcgen05 + TMEM + TMA).
+// Persistent dense tensor-core attention over paged KV (tcgen05 + TMEM + TMA).
 //
-// Level 1 of the decode cascade.  All requests of agent a share the same
-// resident prefix (Sec. I: one static path of the prefix cache per agent;
-// Sec. III, Eq. 2: the prefix is paid once per agent), so the queries of
-// all of a's decode tokens are stacked into 128-row tiles (128/G tokens x G
-// heads of one kv head) and the prefix K/V is streamed through the tensor
-// cores once per tile instead of once per request.  The same kernel runs
-// chunked causal prefill (Sec. VI cites chunked prefill): a tile of one
-// request's chunk attends to the whole prefix and then causally to the
-// request's own suffix.
+// One launch runs a whole list of work items, each a 128-row query tile
+// (128/G tokens x the G q heads of one kv head) against up to two key
+// segments (runs of pages of one prefix or one suffix):
 //
-// One CTA = one work item (a 128-row Q tile against up to two key segments).
+//  * decode, level 1: all requests of agent a share one resident prefix
+//    (Sec. I: one static path of the prefix cache per agent; Sec. III,
+//    Eq. 2: the prefix is paid once per agent), so the queries of all of a's
+//    decode tokens are stacked and the prefix K/V streams through the tensor
+//    cores once per tile instead of once per request;
+//  * decode, level 2: one request's G rows against its own suffix; the item
+//    first appends the step's new token to the pool (the new KV is part of
+//    the request's own state d_r of Eq. 2), then reads it back with the rest
+//    of the suffix;
+//  * decode partials are merged exactly by log-sum-exp inside the kernel:
+//    the item that completes the last partial of a (token, kv head) merges
+//    them (arrival counters in the plan);
+//  * chunked causal prefill (Sec. VI cites chunked prefill): a tile of one
+//    request's chunk attends to the whole prefix and causally to the
+//    request's own suffix, writing final outputs directly.
+//
+// A CTA owns one SM (198 KB of shared memory, 512 TMEM columns) and walks
+// its share of the item list (longest first, snake order over CTAs).
 //   warp 0      TMA producer: K and V tiles (8 pages, one 128B-swizzled box
-//               per page and operand) into a 2-stage ring; lane i loads page
-//               i's id two tiles ahead and issues that page's boxes
-//   warp 1      TMEM owner; one lane issues tcgen05.mma:
+//               per page and operand) into a 2-stage ring, running ahead
+//               across item boundaries; lane i loads page i's id two tiles
+//               ahead and issues that page's boxes
+//   warp 1      TMEM owner; one lane issues tcgen05.mma, whichever of QK /
+//               PV is ready first (QK may run two tiles ahead of PV):
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
 //                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
-//               issuing whichever is ready first (QK may run up to two
-//               tiles ahead of PV), so the softmax of tile j+1 overlaps the
-//               tensor work of tile j
-//   warps 2..9  softmax, two warps per TMEM lane quarter: warp 2+q+4h owns
-//               rows 32q..32q+31 and key half h (64 keys).  Both warps of a
-//               pair compute the full-row max (so their running max agrees
-//               without synchronising), exponentiate their own half in base
-//               2, keep a partial row sum, and write their half of P (bf16)
-//               to shared memory.  O in TMEM is rescaled only when the max
-//               grew by more than 2^8; otherwise the stale max stays the
-//               reference, which is exact (the max is only a stabiliser).
-//               The two partial sums meet once, in the epilogue.
-// Every mbarrier wait is bounded; on a timeout the CTA records a status bit,
-// drains its copies and MMAs, frees TMEM and returns.
+//   warps 2..9  two per TMEM lane quarter: warp 2+q+4h owns rows 32q..32q+31
+//               and key half h.  Per item: load their part of Q, then per
+//               tile read S, take the full-row max (both warps of a pair, so
+//               their running max agrees without synchronising), write P for
+//               their key half, rescale O in TMEM only when the max grew by
+//               more than 2^8 (otherwise the stale max stays the reference,
+//               which is exact: it is only a stabiliser); then the epilogue.
+// Every mbarrier wait is bounded.  On a timeout the CTA records a status bit
+// and every role still walks the same item/tile sequence (skipping the work,
+// never a named barrier), drains its copies and MMAs, frees TMEM and returns.
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -39,6 +48,7 @@ namespace tpa {
 namespace {
 
 constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 constexpr int kThreads = 320;               // producer, MMA, 8 softmax warps
 constexpr int kSoftmax = 256;
@@ -48,6 +58,14 @@ __device__ __forceinline__ float fast_exp2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+
+// Order this thread's generic-proxy global writes before later async-proxy
+// (TMA) reads of the same memory.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+__device__ __forceinline__ void softmax_bar() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
 
 template <int D>
 struct DenseCfg {
@@ -66,7 +84,8 @@ struct DenseCfg {
   static constexpr int kOffBar = kOffV + kStages * kKVBytes;
   static constexpr int kNumBars = 16;
   static constexpr int kOffL = kOffBar + kNumBars * 8;   // partial row sums [2][128]
-  static constexpr int kOffMisc = kOffL + 2 * 128 * 4;
+  static constexpr int kOffFlag = kOffL + 2 * 128 * 4;   // merge flags per token [32]
+  static constexpr int kOffMisc = kOffFlag + 32 * 4;
   static constexpr int kSmem = 1024 + kOffMisc + 64;
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
@@ -74,7 +93,7 @@ struct DenseCfg {
 
 // barrier slots
 enum { B_KFULL = 0, B_KEMPTY = 2, B_VFULL = 4, B_VEMPTY = 6, B_SFULL = 8, B_SFREE = 10,
-       B_PFULL = 12, B_OFULL = 13, B_DRAIN = 14 };
+       B_PFULL = 12, B_OFULL = 13, B_QFULL = 14, B_DRAIN = 15 };
 
 struct TileInfo {
   int key0;     // first key of the tile within its segment
@@ -96,6 +115,12 @@ __device__ __forceinline__ TileInfo tile_at(const DenseItem& it, int j) {
   return t;
 }
 
+// k-th item of this CTA: snake order over CTAs on a longest-first list.
+__device__ __forceinline__ int item_of(int k) {
+  const int g = static_cast<int>(gridDim.x);
+  return k * g + ((k & 1) ? g - 1 - static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x));
+}
+
 template <int D, int G>
 __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constant__ DenseParams p) {
   using C = DenseCfg<D>;
@@ -104,13 +129,12 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kOffBar);
   float* lpart = reinterpret_cast<float*>(smem + C::kOffL);
+  int* mflag = reinterpret_cast<int*>(smem + C::kOffFlag);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const DenseItem item = p.items[blockIdx.x];
-  const int ntiles = item.n_tiles;
 
   // ---------------------------------------------------------------- setup
   if (threadIdx.x == 0) {
@@ -125,6 +149,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     }
     mbar_init(&bars[B_PFULL], kSoftmax);
     mbar_init(&bars[B_OFULL], 1);
+    mbar_init(&bars[B_QFULL], kSoftmax);
     mbar_init(&bars[B_DRAIN], 1);
     fence_mbar_init();
     prefetch_tmap(&p.tmap_k);
@@ -132,37 +157,9 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
-  __syncthreads();  // barriers initialised, TMEM allocated: the producer can start
+  __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
-  // softmax threads: row, key half, token; their slice of the Q row goes to
-  // shared memory while the producer's first K/V loads are in flight
-  const int sw = warp - 2;                 // softmax warp index 0..7
-  const int half = sw >> 2;                // key half (and O column half)
-  const int row = 32 * (warp & 3) + lane;  // TMEM lane quarter = warp % 4
-  const int tok = row / G;
-  const bool row_valid = warp >= 2 && tok < item.n_tok;
-  DenseTok dt = {0, 0x7fffffff, 0, 0};
-  if (row_valid) dt = p.toks[item.tok_base + tok];
-  const int head = item.kv_head * G + row % G;
-  if (warp >= 2) {
-    constexpr int U = D / 16;  // 16-byte units of this thread's half row
-    uint8_t* qs = smem + C::kOffQ;
-    const uint4* src = reinterpret_cast<const uint4*>(
-        p.q + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D) + half * U;
-    uint4 v[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) v[u] = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int gu = half * U + u;
-      *reinterpret_cast<uint4*>(qs + (gu >> 3) * C::kChunk + swz128(row, gu & 7)) = v[u];
-    }
-    fence_proxy_async();
-  }
-  // Q is complete before the MMA warp issues the first QK (softmax warps + MMA warp)
-  if (warp >= 1) asm volatile("bar.sync 1, 288;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -171,42 +168,67 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     // lanes at once.  Lane 0 posts the expected byte count first.
     int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
     bool pok = true;
-    // this lane's page id of tile j (raw; validated when used, two tiles later)
-    auto page_id = [&](int j) -> int32_t {
-      if (j >= ntiles) return 0;
-      const TileInfo t = tile_at(item, j);
-      return lane < (t.nvalid + kPage - 1) / kPage ? __ldg(p.pages + t.page_off + lane) : 0;
-    };
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
       return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
     };
-    int32_t pid0 = page_id(0), pid1 = page_id(1);
-    for (int j = 0; j < ntiles; ++j) {
-      const TileInfo t = tile_at(item, j);
-      const int s = j & 1;
-      const uint32_t ph = (j >> 1) & 1;
-      const int npg = (t.nvalid + kPage - 1) / kPage;
-      const uint32_t bytes = static_cast<uint32_t>(npg * C::NCH * 2048);
-      const int32_t pid = pid0;
-      pid0 = pid1;
-      pid1 = page_id(j + 2);
-      const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
-      if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
-      const int z = (bad ? 0 : pid) * p.hkv + item.kv_head;
-      if (!wait_all(&bars[B_KEMPTY + s], ph ^ 1u)) { pok = false; break; }
-      if (lane == 0) mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
-      __syncwarp();
-      if (lane < npg)
-        tma_load_5d(smem + C::kOffK + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_k,
-                    &bars[B_KFULL + s], 0, 0, 0, 0, z);
-      kph_last[s] = static_cast<int>(ph);
-      if (!wait_all(&bars[B_VEMPTY + s], ph ^ 1u)) { pok = false; break; }
-      if (lane == 0) mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
-      __syncwarp();
-      if (lane < npg)
-        tma_load_5d(smem + C::kOffV + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_v,
-                    &bars[B_VFULL + s], 0, 0, 0, 0, z);
-      vph_last[s] = static_cast<int>(ph);
+    int gt = 0;  // tiles of this CTA so far (ring position)
+    for (int k = 0; pok; ++k) {
+      const int idx = item_of(k);
+      if (idx >= p.n_items) break;
+      const DenseItem item = p.items[idx];
+      const int ntiles = item.n_tiles;
+      if (item.app_src >= 0) {
+        // append the step's token to the pool before any key of it is loaded
+        constexpr int U = D / 8;  // 16-byte units of one row
+        const int64_t src = (static_cast<int64_t>(item.app_src) * p.hkv + item.kv_head) * D;
+        const int64_t pg = item.app_dst / kPage;
+        const int64_t dst = ((pg * p.hkv + item.kv_head) * kPage + item.app_dst % kPage) * D;
+        if (pg >= 0 && pg < p.num_pages) {
+          for (int u = lane; u < 2 * U; u += 32) {
+            const bool isv = u >= U;
+            const int uu = isv ? u - U : u;
+            const uint4 v = reinterpret_cast<const uint4*>((isv ? p.v_new : p.k_new) + src)[uu];
+            reinterpret_cast<uint4*>((isv ? p.v_pool : p.k_pool) + dst)[uu] = v;
+          }
+        } else if (lane == 0) {
+          atomicOr(p.status, kStatusBadPage);
+        }
+        fence_proxy_async_global();
+        __syncwarp();
+      }
+      auto page_id = [&](int j) -> int32_t {  // raw; validated when used
+        if (j >= ntiles) return 0;
+        const TileInfo t = tile_at(item, j);
+        return lane < (t.nvalid + kPage - 1) / kPage ? __ldg(p.pages + t.page_off + lane) : 0;
+      };
+      int32_t pid0 = page_id(0), pid1 = page_id(1);
+      for (int j = 0; j < ntiles; ++j, ++gt) {
+        const TileInfo t = tile_at(item, j);
+        const int s = gt & 1;
+        const uint32_t ph = (gt >> 1) & 1;
+        const int npg = (t.nvalid + kPage - 1) / kPage;
+        const uint32_t bytes = static_cast<uint32_t>(npg * C::kPageBytes);
+        const int32_t pid = pid0;
+        pid0 = pid1;
+        pid1 = page_id(j + 2);
+        const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
+        if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
+        const int z = (bad ? 0 : pid) * p.hkv + item.kv_head;
+        if (!wait_all(&bars[B_KEMPTY + s], ph ^ 1u)) { pok = false; break; }
+        if (lane == 0) mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
+        __syncwarp();
+        if (lane < npg)
+          tma_load_5d(smem + C::kOffK + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_k,
+                      &bars[B_KFULL + s], 0, 0, 0, 0, z);
+        kph_last[s] = static_cast<int>(ph);
+        if (!wait_all(&bars[B_VEMPTY + s], ph ^ 1u)) { pok = false; break; }
+        if (lane == 0) mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
+        __syncwarp();
+        if (lane < npg)
+          tma_load_5d(smem + C::kOffV + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_v,
+                      &bars[B_VFULL + s], 0, 0, 0, 0, z);
+        vph_last[s] = static_cast<int>(ph);
+      }
     }
     if (!pok && lane == 0) {
       *abort_flag = 1;
@@ -230,8 +252,8 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       const uint32_t pbase = smem_u32(smem + C::kOffP);
       const uint32_t kbase0 = smem_u32(smem + C::kOffK);
       const uint32_t vbase0 = smem_u32(smem + C::kOffV);
-      auto issue_qk = [&](int j) {
-        const int s = j & 1;
+      auto issue_qk = [&](int g) {
+        const int s = g & 1;
         tc_fence_after();
         const uint32_t kb = kbase0 + s * C::kKVBytes;
         const uint32_t scol = s ? C::kColS1 : C::kColS0;
@@ -244,47 +266,61 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         umma_commit(&bars[B_SFULL + s]);
         umma_commit(&bars[B_KEMPTY + s]);
       };
-      auto issue_pv = [&](int i) {
-        const int s = i & 1;
+      auto issue_pv = [&](int g, bool first) {
+        const int s = g & 1;
         tc_fence_after();
         const uint32_t vb = vbase0 + s * C::kKVBytes;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint64_t a = umma_sdesc(pbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
           const uint64_t b = umma_sdesc(vb + kk * C::kPageBytes, 1024, C::kGroup);
-          umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+          umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (!first || kk > 0) ? 1u : 0u);
         }
         umma_commit(&bars[B_OFULL]);
         umma_commit(&bars[B_VEMPTY + s]);
       };
-      // Issue whichever is ready first: QK of the next tile (K landed, its S
-      // buffer released by the softmax two tiles back) or PV of the oldest
-      // tile whose P is written (and V landed).  PVs stay in tile order.
       bool ok = true;
-      int nq = 0, np = 0;
-      unsigned long long t_last = global_ns();
-      while (ok && np < ntiles) {
-        bool progressed = false;
-        if (nq < ntiles && nq <= np + 2) {
-          const int s = nq & 1;
-          const uint32_t ph = (nq >> 1) & 1;
-          if (mbar_test(&bars[B_KFULL + s], ph) && mbar_test(&bars[B_SFREE + s], ph ^ 1u)) {
-            issue_qk(nq++);
-            progressed = true;
+      int gt = 0;
+      for (int k = 0; ok; ++k) {
+        const int idx = item_of(k);
+        if (idx >= p.n_items) break;
+        const int ntiles = p.items[idx].n_tiles;
+        // Q of this item is written by the softmax warps only after the
+        // previous item's last PV completed (so Q and O are free again)
+        if (!mbar_wait(&bars[B_QFULL], k & 1, abort_flag)) { ok = false; break; }
+        // Issue whichever is ready first: QK of the next tile (K landed, its S
+        // buffer released by the softmax two tiles back) or PV of the oldest
+        // tile whose P is written (and V landed).  PVs stay in tile order.
+        int nq = 0, np = 0;
+        unsigned long long t_last = global_ns();
+        while (ok && np < ntiles) {
+          bool progressed = false;
+          if (nq < ntiles && nq <= np + 2) {
+            const int g = gt + nq;
+            const int s = g & 1;
+            const uint32_t ph = (g >> 1) & 1;
+            if (mbar_test(&bars[B_KFULL + s], ph) && mbar_test(&bars[B_SFREE + s], ph ^ 1u)) {
+              issue_qk(g);
+              ++nq;
+              progressed = true;
+            }
+          }
+          if (np < nq) {
+            const int g = gt + np;
+            if (mbar_test(&bars[B_PFULL], g & 1) &&
+                mbar_test(&bars[B_VFULL + (g & 1)], (g >> 1) & 1)) {
+              issue_pv(g, np == 0);
+              ++np;
+              progressed = true;
+            }
+          }
+          if (progressed) {
+            t_last = global_ns();
+          } else if (*abort_flag || global_ns() - t_last > kWaitLimitNs) {
+            ok = false;
           }
         }
-        if (np < nq) {
-          const int s = np & 1;
-          if (mbar_test(&bars[B_PFULL], np & 1) && mbar_test(&bars[B_VFULL + s], (np >> 1) & 1)) {
-            issue_pv(np++);
-            progressed = true;
-          }
-        }
-        if (progressed) {
-          t_last = global_ns();
-        } else if (*abort_flag || global_ns() - t_last > kWaitLimitNs) {
-          ok = false;
-        }
+        gt += ntiles;
       }
       if (!ok) {
         *abort_flag = 1;
@@ -297,143 +333,183 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     }
   } else {
     // ------------------------------------------------------------ softmax
+    // Every softmax thread walks the same items and tiles even after a
+    // failure (ok == false skips the work): the named barriers below must be
+    // reached the same number of times by all 256 threads.
+    const int sw = warp - 2;                 // softmax warp index 0..7
+    const int half = sw >> 2;                // key half (and O column half)
+    const int row = 32 * (warp & 3) + lane;  // TMEM lane quarter = warp % 4
+    const int tok = row / G;
     const uint32_t lane_base = static_cast<uint32_t>(32 * (warp & 3)) << 16;
     const int own = half * 64;   // first S column of this thread's key half
     const int other = 64 - own;
     const float sc = p.scale_log2;
     uint8_t* ps = smem + C::kOffP;
-    float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     // warp-uniform outcome, so .sync.aligned tcgen05 ops never see a split warp
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
-      return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
+      if (!ok) return false;
+      if (__all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag))) return true;
+      *abort_flag = 1;  // let the other roles stop waiting too
+      return false;
     };
-    for (int j = 0; j < ntiles; ++j) {
-      const TileInfo t = tile_at(item, j);
-      const int s = j & 1;
-      if (!wait_all(&bars[B_SFULL + s], (j >> 1) & 1)) { ok = false; break; }
-      tc_fence_after();
-      const uint32_t scol = tmem + lane_base + (s ? C::kColS1 : C::kColS0);
-      float x[64], y[64];
-      tmem_ld32(scol + own, x);
-      tmem_ld32(scol + own + 32, x + 32);
-      tmem_ld32(scol + other, y);
-      tmem_ld32(scol + other + 32, y + 32);
-      tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(&bars[B_SFREE + s]);
-
-      int lim = t.nvalid;
-      if (t.causal && dt.causal_pos < t.key0 + lim) {
-        const int c = dt.causal_pos - t.key0 + 1;
-        lim = c > 0 ? c : 0;
-      }
-      if (lim < 128) {
+    int gt = 0;
+    for (int k = 0;; ++k) {
+      const int idx = item_of(k);
+      if (idx >= p.n_items) break;
+      const DenseItem item = p.items[idx];
+      const int ntiles = item.n_tiles;
+      const bool row_valid = tok < item.n_tok;
+      DenseTok dt = {0, 0x7fffffff, 0, 0};
+      if (row_valid) dt = p.toks[item.tok_base + tok];
+      const int head = item.kv_head * G + row % G;
+      {
+        // this thread's half of its Q row (zero for padding rows)
+        constexpr int U = D / 16;
+        uint8_t* qs = smem + C::kOffQ;
+        const uint4* src = reinterpret_cast<const uint4*>(
+            p.q + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D) + half * U;
+        uint4 v[U];
 #pragma unroll
-        for (int n = 0; n < 64; ++n) {
-          x[n] = own + n < lim ? x[n] : -INFINITY;
-          y[n] = other + n < lim ? y[n] : -INFINITY;
+        for (int u = 0; u < U; ++u) v[u] = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int gu = half * U + u;
+          *reinterpret_cast<uint4*>(qs + (gu >> 3) * C::kChunk + swz128(row, gu & 7)) = v[u];
         }
+        fence_proxy_async();
+        mbar_arrive(&bars[B_QFULL]);
       }
-      // full-row max of the raw scores: 8 independent chains of 3-input max
-      float acc[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) acc[i] = fmax3f(x[i], x[i + 8], y[i]);
-#pragma unroll
-      for (int k = 16; k < 64; k += 8)
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], x[k + i], y[k + i - 8]);
-#pragma unroll
-      for (int i = 0; i < 8; ++i) acc[i] = fmaxf(acc[i], y[56 + i]);
-      const float mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
-                                fmaxf(acc[6], acc[7]));
-      const float mx = mraw * sc;  // sc > 0: max of the scaled scores
-      const float m_new = fmaxf(m_run, mx);
-      const bool grow = m_new > m_run + kRescaleThreshold;
-      const float m_use = grow ? m_new : m_run;
-      const float alpha = grow ? fast_exp2(m_run - m_use) : 1.f;
-      const float nref = m_use == -INFINITY ? 0.f : -m_use;
-      // p = 2^(s * sc - m) over this thread's half: packed FMAs, MUFU ex2,
-      // 8 independent partial sums
-      float sacc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int n = 0; n < 64; n += 2) {
-        ffma2(x[n], x[n + 1], x[n], x[n + 1], sc, sc, nref, nref);
-        x[n] = fast_exp2(x[n]);
-        x[n + 1] = fast_exp2(x[n + 1]);
-      }
-#pragma unroll
-      for (int n = 0; n < 64; n += 16)
-#pragma unroll
-        for (int i = 0; i < 8; i += 2) {
-          fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i], x[n + 2 * i + 1]);
-          fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i + 2], x[n + 2 * i + 3]);
-        }
-      const float rsum = ((sacc[0] + sacc[1]) + (sacc[2] + sacc[3])) +
-                         ((sacc[4] + sacc[5]) + (sacc[6] + sacc[7]));
-      if (j > 0) {
-        if (!wait_all(&bars[B_OFULL], (j - 1) & 1)) { ok = false; break; }
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; j < ntiles && ok; ++j) {
+        const TileInfo t = tile_at(item, j);
+        const int g = gt + j;
+        const int s = g & 1;
+        if (!wait_all(&bars[B_SFULL + s], (g >> 1) & 1)) { ok = false; break; }
         tc_fence_after();
-        // rescale this half of the O row when the reference max moved (with real content)
-        const bool need = grow && m_run > -INFINITY;
-        if (__any_sync(0xffffffffu, need)) {
+        const uint32_t scol = tmem + lane_base + (s ? C::kColS1 : C::kColS0);
+        float x[64], y[64];
+        tmem_ld32(scol + own, x);
+        tmem_ld32(scol + own + 32, x + 32);
+        tmem_ld32(scol + other, y);
+        tmem_ld32(scol + other + 32, y + 32);
+        tmem_wait_ld();
+        tc_fence_before();
+        mbar_arrive(&bars[B_SFREE + s]);
+
+        int lim = t.nvalid;
+        if (t.causal && dt.causal_pos < t.key0 + lim) {
+          const int c = dt.causal_pos - t.key0 + 1;
+          lim = c > 0 ? c : 0;
+        }
+        if (lim < 128) {
+#pragma unroll
+          for (int n = 0; n < 64; ++n) {
+            x[n] = own + n < lim ? x[n] : -INFINITY;
+            y[n] = other + n < lim ? y[n] : -INFINITY;
+          }
+        }
+        // full-row max of the raw scores: 8 independent chains of 3-input max
+        float acc[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = fmax3f(x[i], x[i + 8], y[i]);
+#pragma unroll
+        for (int kk = 16; kk < 64; kk += 8)
+#pragma unroll
+          for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], x[kk + i], y[kk + i - 8]);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = fmaxf(acc[i], y[56 + i]);
+        const float mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
+                                  fmaxf(acc[6], acc[7]));
+        const float mx = mraw * sc;  // sc > 0: max of the scaled scores
+        const float m_new = fmaxf(m_run, mx);
+        const bool grow = m_new > m_run + kRescaleThreshold;
+        const float m_use = grow ? m_new : m_run;
+        const float alpha = grow ? fast_exp2(m_run - m_use) : 1.f;
+        const float nref = m_use == -INFINITY ? 0.f : -m_use;
+        // p = 2^(s * sc - m) over this thread's half: packed FMAs, MUFU ex2,
+        // 8 independent partial sums
+        float sacc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int n = 0; n < 64; n += 2) {
+          ffma2(x[n], x[n + 1], x[n], x[n + 1], sc, sc, nref, nref);
+          x[n] = fast_exp2(x[n]);
+          x[n + 1] = fast_exp2(x[n + 1]);
+        }
+#pragma unroll
+        for (int n = 0; n < 64; n += 16)
+#pragma unroll
+          for (int i = 0; i < 8; i += 2) {
+            fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i], x[n + 2 * i + 1]);
+            fadd2(sacc[i], sacc[i + 1], sacc[i], sacc[i + 1], x[n + 2 * i + 2], x[n + 2 * i + 3]);
+          }
+        const float rsum = ((sacc[0] + sacc[1]) + (sacc[2] + sacc[3])) +
+                           ((sacc[4] + sacc[5]) + (sacc[6] + sacc[7]));
+        if (j > 0) {
+          if (!wait_all(&bars[B_OFULL], (g - 1) & 1)) { ok = false; break; }
+          tc_fence_after();
+          // rescale this half of the O row when the reference max moved (with real content)
+          const bool need = grow && m_run > -INFINITY;
+          if (__any_sync(0xffffffffu, need)) {
 #pragma unroll 1
-          for (int c = 0; c < D / 64; ++c) {
-            float o[32];
-            const uint32_t oc = tmem + lane_base + C::kColO + half * (D / 2) + 32 * c;
-            tmem_ld32(oc, o);
-            tmem_wait_ld();
+            for (int c = 0; c < D / 64; ++c) {
+              float o[32];
+              const uint32_t oc = tmem + lane_base + C::kColO + half * (D / 2) + 32 * c;
+              tmem_ld32(oc, o);
+              tmem_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] *= alpha;
-            tmem_st32(oc, o);
-          }
-          tmem_wait_st();
-        }
-      }
-      l_run = l_run * alpha + rsum;
-      m_run = m_use;
-      if (t.nvalid < 128) {
-        // keys past the range: zero their V rows (stale data may not be finite);
-        // each half zeroes its own 64-dim chunk (or its half of the only chunk)
-        if (!wait_all(&bars[B_VFULL + s], (j >> 1) & 1)) { ok = false; break; }
-        if (row >= t.nvalid) {
-          uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
-          if (C::NCH == 2) {
-#pragma unroll
-            for (int u = 0; u < 8; ++u)
-              *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(row, 8 * half + u)) =
-                  make_uint4(0, 0, 0, 0);
-          } else {
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-              *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(row, 4 * half + u)) =
-                  make_uint4(0, 0, 0, 0);
+              for (int i = 0; i < 32; ++i) o[i] *= alpha;
+              tmem_st32(oc, o);
+            }
+            tmem_wait_st();
           }
         }
-      }
-      // this half of the P row: keys own .. own+63 = P chunk `half`
+        l_run = l_run * alpha + rsum;
+        m_run = m_use;
+        if (t.nvalid < 128) {
+          // keys past the range: zero their V rows (stale data may not be finite);
+          // each half zeroes its own 64-dim chunk (or its half of the only chunk)
+          if (!wait_all(&bars[B_VFULL + s], (g >> 1) & 1)) { ok = false; break; }
+          if (row >= t.nvalid) {
+            uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
+            if (C::NCH == 2) {
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        uint4 v;
-        v.x = pack_bf16(x[8 * u + 0], x[8 * u + 1]);
-        v.y = pack_bf16(x[8 * u + 2], x[8 * u + 3]);
-        v.z = pack_bf16(x[8 * u + 4], x[8 * u + 5]);
-        v.w = pack_bf16(x[8 * u + 6], x[8 * u + 7]);
-        *reinterpret_cast<uint4*>(ps + half * C::kChunk + swz128(row, u)) = v;
+              for (int u = 0; u < 8; ++u)
+                *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(row, 8 * half + u)) =
+                    make_uint4(0, 0, 0, 0);
+            } else {
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(row, 4 * half + u)) =
+                    make_uint4(0, 0, 0, 0);
+            }
+          }
+        }
+        // this half of the P row: keys own .. own+63 = P chunk `half`
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          uint4 v;
+          v.x = pack_bf16(x[8 * u + 0], x[8 * u + 1]);
+          v.y = pack_bf16(x[8 * u + 2], x[8 * u + 3]);
+          v.z = pack_bf16(x[8 * u + 4], x[8 * u + 5]);
+          v.w = pack_bf16(x[8 * u + 6], x[8 * u + 7]);
+          *reinterpret_cast<uint4*>(ps + half * C::kChunk + swz128(row, u)) = v;
+        }
+        fence_proxy_async();
+        tc_fence_before();
+        mbar_arrive(&bars[B_PFULL]);
       }
-      fence_proxy_async();
-      tc_fence_before();
-      mbar_arrive(&bars[B_PFULL]);
-    }
-    // combine the two halves' partial row sums
-    lpart[half * 128 + row] = l_run;
-    asm volatile("bar.sync 2, 256;" ::: "memory");
-    const float l_tot = lpart[row] + lpart[128 + row];
-    if (ok && ntiles > 0) {
-      ok = wait_all(&bars[B_OFULL], (ntiles - 1) & 1);
+
+      // ---------------------------------------------------------- epilogue
+      lpart[half * 128 + row] = l_run;
+      softmax_bar();
+      const float l_tot = lpart[row] + lpart[128 + row];
+      if (!wait_all(&bars[B_OFULL], (gt + ntiles - 1) & 1)) ok = false;
+      const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
+      const float lse = l_tot > 0.f ? (m_run + __log2f(l_tot)) * kLn2 : -INFINITY;
+      const int64_t slot = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
       if (ok) {
         tc_fence_after();
-        const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
 #pragma unroll 1
         for (int c = 0; c < D / 64; ++c) {
           float o[32];
@@ -442,8 +518,6 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           tmem_wait_ld();
           if (row_valid) {
             if (item.out_mode == 0) {
-              const int64_t slot =
-                  dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
               float4* dst = reinterpret_cast<float4*>(p.part_o + slot * D + col);
 #pragma unroll
               for (int i = 0; i < 8; ++i)
@@ -464,16 +538,68 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
             }
           }
         }
+        tc_fence_before();
         if (row_valid && half == 0) {
-          const float lse = l_tot > 0.f ? (m_run + __log2f(l_tot)) * kLn2 : -INFINITY;
-          if (item.out_mode == 0) {
-            const int64_t slot = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
-            p.part_lse[slot] = lse;
-          } else {
-            p.lse[static_cast<int64_t>(dt.q_row) * p.hq + head] = lse;
-          }
+          if (item.out_mode == 0) p.part_lse[slot] = lse;
+          else p.lse[static_cast<int64_t>(dt.q_row) * p.hq + head] = lse;
         }
       }
+      if (item.out_mode == 0 && p.counters) {
+        // the item that completes the last partial of a (token, kv head)
+        // merges all of them: o = sum c_i o_i / sum c_i, c_i = e^(lse_i - M)
+        __threadfence();
+        softmax_bar();
+        if (half == 0 && row % G == 0) {
+          int last = 0;
+          if (row_valid && ok) {
+            const uint32_t prev = atomicAdd(
+                p.counters + static_cast<int64_t>(dt.q_row) * p.hkv + item.kv_head, 1u);
+            last = prev + 1 == static_cast<uint32_t>(dt.n_slots);
+          }
+          mflag[tok] = last;
+        }
+        softmax_bar();
+        if (row_valid && mflag[tok]) {
+          __threadfence();
+          const int64_t base = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots;
+          float mxl = -INFINITY;
+          for (int i = 0; i < dt.n_slots; ++i) mxl = fmaxf(mxl, __ldcg(p.part_lse + base + i));
+          float macc[D / 2];
+#pragma unroll
+          for (int c = 0; c < D / 2; ++c) macc[c] = 0.f;
+          float tot = 0.f;
+          for (int i = 0; i < dt.n_slots; ++i) {
+            const float w = exp2f((__ldcg(p.part_lse + base + i) - mxl) * kLog2e);
+            tot += w;
+            const float4* src =
+                reinterpret_cast<const float4*>(p.part_o + (base + i) * D + half * (D / 2));
+#pragma unroll
+            for (int c = 0; c < D / 8; ++c) {
+              const float4 v = __ldcg(src + c);
+              macc[4 * c] += w * v.x;
+              macc[4 * c + 1] += w * v.y;
+              macc[4 * c + 2] += w * v.z;
+              macc[4 * c + 3] += w * v.w;
+            }
+          }
+          const float itot = tot > 0.f ? 1.f / tot : 0.f;
+          uint4* dst = reinterpret_cast<uint4*>(
+              p.out + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D + half * (D / 2));
+#pragma unroll
+          for (int c = 0; c < D / 16; ++c) {
+            uint4 v;
+            v.x = pack_bf16(macc[8 * c + 0] * itot, macc[8 * c + 1] * itot);
+            v.y = pack_bf16(macc[8 * c + 2] * itot, macc[8 * c + 3] * itot);
+            v.z = pack_bf16(macc[8 * c + 4] * itot, macc[8 * c + 5] * itot);
+            v.w = pack_bf16(macc[8 * c + 6] * itot, macc[8 * c + 7] * itot);
+            dst[c] = v;
+          }
+          if (half == 0)
+            p.lse[static_cast<int64_t>(dt.q_row) * p.hq + head] =
+                tot > 0.f ? mxl + __log2f(tot) * kLn2 : -INFINITY;
+        }
+      }
+      gt += ntiles;
     }
     if (!ok) {
       *abort_flag = 1;
@@ -491,20 +617,21 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 }
 
 template <int D, int G>
-cudaError_t launch_dense_t(const DenseParams& p, int n_items, cudaStream_t stream) {
-  dense_kernel<D, G><<<n_items, kThreads, DenseCfg<D>::kSmem, stream>>>(p);
+cudaError_t launch_dense_t(const DenseParams& p, int num_sms, cudaStream_t stream) {
+  const int grid = p.n_items < num_sms ? p.n_items : num_sms;
+  dense_kernel<D, G><<<grid, kThreads, DenseCfg<D>::kSmem, stream>>>(p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_dense(const DenseParams& p, int n_items, int head_dim, int group,
+cudaError_t launch_dense(const DenseParams& p, int num_sms, int head_dim, int group,
                          cudaStream_t stream) {
-  if (n_items <= 0) return cudaSuccess;
-  if (head_dim == 128 && group == 4) return launch_dense_t<128, 4>(p, n_items, stream);
-  if (head_dim == 128 && group == 8) return launch_dense_t<128, 8>(p, n_items, stream);
-  if (head_dim == 64 && group == 4) return launch_dense_t<64, 4>(p, n_items, stream);
-  if (head_dim == 64 && group == 8) return launch_dense_t<64, 8>(p, n_items, stream);
+  if (p.n_items <= 0) return cudaSuccess;
+  if (head_dim == 128 && group == 4) return launch_dense_t<128, 4>(p, num_sms, stream);
+  if (head_dim == 128 && group == 8) return launch_dense_t<128, 8>(p, num_sms, stream);
+  if (head_dim == 64 && group == 4) return launch_dense_t<64, 4>(p, num_sms, stream);
+  if (head_dim == 64 && group == 8) return launch_dense_t<64, 8>(p, num_sms, stream);
   return cudaErrorInvalidValue;
 }
 

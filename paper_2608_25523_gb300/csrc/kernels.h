@@ -41,14 +41,21 @@ struct DenseParams {
   const DenseItem* items;
   const DenseTok* toks;
   const int32_t* pages;
+  const __nv_bfloat16* k_new;  // rows appended by items with app_src >= 0
+  const __nv_bfloat16* v_new;
+  __nv_bfloat16* k_pool;
+  __nv_bfloat16* v_pool;
+  uint32_t* counters;  // zeroed [q rows][hkv] arrival counts; non-null: merge partials in-kernel
   uint32_t* status;
   int64_t num_pages;
+  int n_items;
   int hq, hkv;
   float scale_log2;  // log2(e) / sqrt(d)
 };
 
-// Dense tensor-core attention of 128-row query tiles (tcgen05 + TMEM + TMA).
-cudaError_t launch_dense(const DenseParams& p, int n_items, int head_dim, int group,
+// Persistent dense tensor-core attention over a list of 128-row query tiles
+// (tcgen05 + TMEM + TMA), one CTA per SM at most.
+cudaError_t launch_dense(const DenseParams& p, int num_sms, int head_dim, int group,
                          cudaStream_t stream);
 
 struct SuffixParams {

@@ -44,7 +44,8 @@ struct DenseItem {
   int32_t seg_k0[2];      // first key of the range (multiple of 16)
   int32_t seg_k1[2];      // one past the last key of the range (k1 == k0: empty)
   int32_t seg_causal[2];  // 1: causal mask on this segment
-  int32_t pad[2];
+  int32_t app_src;        // decode: row of k_new/v_new appended before the keys are read (-1: none)
+  int32_t app_dst;        // page * 16 + slot the appended row goes to
 };
 static_assert(sizeof(DenseItem) == 64, "DenseItem layout");
 
@@ -72,8 +73,8 @@ struct MergeTok {
 
 // Header of an uploaded plan blob; offsets in bytes from the blob start.
 struct PlanHeader {
-  int32_t n_pages, n_append, n_dense_tok, n_dense, n_suffix, n_merge;
-  int32_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge;
+  int32_t n_pages, n_append, n_dense_tok, n_dense, n_suffix, n_merge, n_counters;
+  int32_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, off_counters;
   uint32_t queue[4];  // zero on upload: atomic work counters of persistent kernels
 };
 
