@@ -56,6 +56,7 @@ int fail(int code, const char* fmt, ...) {
   } while (0)
 
 constexpr int kRingSlots = 4;
+constexpr int kSplitWarpsPerCta = 8;  // split-KV warps of a CTA in the fused decode launch
 constexpr int kKernelKinds = 5;  // append, dense, split-KV, merge, page copy
 enum { K_APPEND = 0, K_DENSE = 1, K_SUFFIX = 2, K_MERGE = 3, K_COPY = 4 };
 constexpr size_t kAlign = 256;
@@ -934,25 +935,32 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       split_keys *= 2;
     }
   } else {
-    // total key tiles over both levels; aim for items of about one SM's share
-    int64_t tiles = 0;
+    // Level 1 (dense role): stacked prefix tiles; split each agent's prefix
+    // so the dense items number about the dense CTAs' count or more.
+    int64_t dense_units = 0;
     for (auto& g : groups)
-      tiles += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) *
-               cdiv(ctx->agents[g.agent].len, kTileKeys);
-    for (int i = 0; i < n; ++i) tiles += hkv * cdiv(keys_of(i), kTileKeys);
-    const int64_t target = std::max<int64_t>(4, cdiv(tiles, ctx->num_sms));
+      if (ctx->agents[g.agent].len > 0)
+        dense_units += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt);
     for (auto& g : groups) {
       const int64_t ptiles = cdiv(ctx->agents[g.agent].len, kTileKeys);
       if (ptiles == 0) continue;
-      int64_t ns = ctx->prefix_splits > 0 ? ctx->prefix_splits : cdiv(ptiles, target);
+      int64_t ns = ctx->prefix_splits > 0 ? ctx->prefix_splits
+                                           : cdiv(ctx->num_sms / 4, std::max<int64_t>(1, dense_units));
       ns = std::min<int64_t>(std::max<int64_t>(ns, 1), ptiles);
       g.tiles_per_split = static_cast<int32_t>(cdiv(ptiles, ns));
       g.n_split = static_cast<int32_t>(cdiv(ptiles, g.tiles_per_split));
       if (g.n_split >= ctx->max_splits)
         return fail(TPA_ERR_CAPACITY, "prefix splits exceed max_splits");
     }
-    split_keys = ctx->suffix_split_keys > 0 ? ctx->suffix_split_keys : target * kTileKeys;
-    split_keys = cdiv(split_keys, kTileKeys) * kTileKeys;
+    // Level 2 (split-KV role): about two items per split-KV warp, 64..1024 keys
+    int64_t sum_keys = 0;
+    for (int i = 0; i < n; ++i) sum_keys += keys_of(i);
+    split_keys = ctx->suffix_split_keys;
+    if (split_keys <= 0) {
+      const int64_t warps = static_cast<int64_t>(ctx->num_sms) * 6;
+      split_keys = std::min<int64_t>(std::max<int64_t>(cdiv(sum_keys * hkv, 2 * warps), 64), 1024);
+    }
+    split_keys = cdiv(split_keys, kPage) * kPage;
     for (;;) {
       int64_t worst = 0;
       for (int i = 0; i < n; ++i)
@@ -984,10 +992,10 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     for (int i = 0; i < n; ++i)
       sz.suffix += hkv * (cdiv(keys_of(i), split_keys) + cdiv(lp_of(i), split_keys));
   } else {
-    sz.dense_tok = 2 * n;
+    sz.dense_tok = n;
     sz.counters = static_cast<int64_t>(n) * hkv;
     for (auto& g : groups) sz.dense += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) * g.n_split;
-    for (int i = 0; i < n; ++i) sz.dense += hkv * cdiv(keys_of(i), split_keys);
+    for (int i = 0; i < n; ++i) sz.suffix += hkv * cdiv(keys_of(i), split_keys);
   }
   const PlanLayout lay = layout_of(sz);
   if (lay.total > ctx->plan_cap)
@@ -1031,7 +1039,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
           for (int h = 0; h < hkv; ++h)
             w.suffix[ns++] = SuffixItem{i, h, static_cast<int32_t>(base + k0 / kPage),
                                         static_cast<int32_t>(std::min<int64_t>(split_keys, len - k0)),
-                                        slot_base[i], n_slots[i], split, 0};
+                                        slot_base[i], n_slots[i], split, -1, 0, {0, 0, 0}};
       }
     }
     std::stable_sort(w.suffix, w.suffix + ns,
@@ -1064,41 +1072,31 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
             it.seg_k1[0] = static_cast<int32_t>(
                 std::min<int64_t>(lp, static_cast<int64_t>(sp + 1) * g.tiles_per_split * kTileKeys));
             it.n_tiles = static_cast<int32_t>(cdiv(it.seg_k1[0] - it.seg_k0[0], kTileKeys));
-            it.app_src = -1;
             w.dense[nd++] = it;
           }
       }
     }
-    // level 2: each token's suffix per kv head; the item holding the last key
-    // appends the step's token first
+    // level 2: each token's suffix per kv head on the split-KV role; the item
+    // holding the last key appends the step's token first
     for (int i = 0; i < n; ++i) {
       const Request& r = ctx->reqs[reqs[i]];
-      const int32_t tok_idx = nt;
-      w.dtok[nt++] = DenseTok{i, 0x7fffffff, slot_base[i], n_slots[i]};
       const int64_t keys = keys_of(i);
       const int pos = r.len;  // slot of the new token
       const int32_t app_dst = r.pages[pos / kPage] * kPage + pos % kPage;
       int split = groups[group_of[i]].n_split;
-      for (int64_t k0 = 0; k0 < keys; k0 += split_keys, ++split)
-        for (int h = 0; h < hkv; ++h) {
-          DenseItem it{};
-          it.tok_base = tok_idx;
-          it.n_tok = 1;
-          it.kv_head = h;
-          it.split = split;
-          it.out_mode = 0;
-          it.seg_pages[0] = suf_off[i];
-          it.seg_k0[0] = static_cast<int32_t>(k0);
-          it.seg_k1[0] = static_cast<int32_t>(std::min<int64_t>(keys, k0 + split_keys));
-          it.n_tiles = static_cast<int32_t>(cdiv(it.seg_k1[0] - it.seg_k0[0], kTileKeys));
-          const bool last = k0 + split_keys >= keys;
-          it.app_src = last ? i : -1;
-          it.app_dst = last ? app_dst : 0;
-          w.dense[nd++] = it;
-        }
+      for (int64_t k0 = 0; k0 < keys; k0 += split_keys, ++split) {
+        const bool last = k0 + split_keys >= keys;
+        for (int h = 0; h < hkv; ++h)
+          w.suffix[ns++] = SuffixItem{i, h, static_cast<int32_t>(suf_off[i] + k0 / kPage),
+                                      static_cast<int32_t>(std::min<int64_t>(split_keys, keys - k0)),
+                                      slot_base[i], n_slots[i], split, last ? i : -1,
+                                      last ? app_dst : 0, {0, 0, 0}};
+      }
     }
     std::stable_sort(w.dense, w.dense + nd,
                      [](const DenseItem& a, const DenseItem& b) { return a.n_tiles > b.n_tiles; });
+    std::stable_sort(w.suffix, w.suffix + ns,
+                     [](const SuffixItem& a, const SuffixItem& b) { return a.n_keys > b.n_keys; });
   }
 
   PlanHeader* hd = w.hdr;
@@ -1151,12 +1149,31 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       }
       launches = 3;
     } else {
+      // one launch, one CTA per SM: dense CTAs for level 1, the rest split-KV;
+      // SMs shared in proportion to estimated time (a dense 128x128 tile
+      // ~1.15 us; split-KV ~35 GB/s of KV per SM)
+      int64_t dense_tiles = 0;
+      for (int i = 0; i < nd; ++i) dense_tiles += w.dense[i].n_tiles;
+      double split_bytes = 0;
+      for (int i = 0; i < ns; ++i) split_bytes += w.suffix[i].n_keys * 4.0 * ctx->d;
+      const double wd = dense_tiles * 1.15, wsplit = split_bytes / 35e3;
+      int n_dense = nd == 0 ? 0 : static_cast<int>(std::lround(ctx->num_sms * wd / (wd + wsplit)));
+      if (nd > 0) n_dense = std::max(n_dense, 1);
+      if (ns > 0) n_dense = std::min(n_dense, ctx->num_sms - 1);
+      n_dense = std::min(n_dense, nd);
+      const int n_split = ns > 0 ? std::min<int>(ctx->num_sms - n_dense,
+                                                 static_cast<int>(cdiv(ns, kSplitWarpsPerCta)))
+                                 : 0;
       DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
+      dp.n_dense_ctas = n_dense;
+      dp.sitems = dev_ptr<SuffixItem>(sl, lay.off_suffix);
+      dp.n_sitems = ns;
+      dp.squeue = reinterpret_cast<uint32_t*>(sl->dev + offsetof(PlanHeader, queue));
       dp.k_new = static_cast<const __nv_bfloat16*>(k_new);
       dp.v_new = static_cast<const __nv_bfloat16*>(v_new);
       dp.counters = reinterpret_cast<uint32_t*>(sl->dev + lay.off_counters);
       KernelTimer kt(ctx, K_DENSE, s);
-      CUDA_TRY(launch_dense(dp, ctx->num_sms, ctx->d, G, s));
+      CUDA_TRY(launch_dense(dp, n_split, ctx->d, G, s));
       launches = 1;
     }
   }
@@ -1187,7 +1204,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   if (total > ctx->cfg.max_tokens) return fail(TPA_ERR_CAPACITY, "%lld tokens > max_tokens", (long long)total);
   if (!ctx->plan_only && (!q || !k_new || !v_new || !out || !lse))
     return fail(TPA_ERR_INVALID_ARG, "null tensor");
-  const int G = ctx->group, hkv = ctx->hkv, hq = ctx->hq;
+  const int G = ctx->group, hkv = ctx->hkv;
   const int tpt = kTileRows / G;
 
   std::vector<int32_t> offset(n);
@@ -1262,7 +1279,6 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
         it.seg_k1[1] = offset[i] + t1;  // keys up to the tile's last position
         it.seg_causal[1] = 1;
         it.n_tiles = static_cast<int32_t>(cdiv(lp, kTileKeys) + cdiv(it.seg_k1[1], kTileKeys));
-        it.app_src = -1;
         w.dense[nd++] = it;
       }
     }
@@ -1288,8 +1304,9 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
                              v_new, ctx->pool, ctx->status, s));
     }
     DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
+    dp.n_dense_ctas = std::min(nd, ctx->num_sms);
     KernelTimer kt(ctx, K_DENSE, s);
-    CUDA_TRY(launch_dense(dp, ctx->num_sms, ctx->d, G, s));
+    CUDA_TRY(launch_dense(dp, 0, ctx->d, G, s));
   }
   for (int i = 0; i < n; ++i) {
     Request& r = ctx->reqs[reqs[i]];

@@ -9,19 +9,18 @@
 //    Eq. 2: the prefix is paid once per agent), so the queries of all of a's
 //    decode tokens are stacked and the prefix K/V streams through the tensor
 //    cores once per tile instead of once per request;
-//  * decode, level 2: one request's G rows against its own suffix; the item
-//    first appends the step's new token to the pool (the new KV is part of
-//    the request's own state d_r of Eq. 2), then reads it back with the rest
-//    of the suffix;
+//  * decode, level 2 runs in the same launch on the other CTAs (split_kv.cuh:
+//    one warp per request suffix range, which also appends the step's token);
 //  * decode partials are merged exactly by log-sum-exp inside the kernel:
-//    the item that completes the last partial of a (token, kv head) merges
-//    them (arrival counters in the plan);
+//    the item (of either role) that completes the last partial of a (token,
+//    kv head) merges them (arrival counters in the plan);
 //  * chunked causal prefill (Sec. VI cites chunked prefill): a tile of one
 //    request's chunk attends to the whole prefix and causally to the
 //    request's own suffix, writing final outputs directly.
 //
-// A CTA owns one SM (198 KB of shared memory, 512 TMEM columns) and walks
-// its share of the item list (longest first, snake order over CTAs).
+// A CTA owns one SM (198 KB of shared memory).  The first n_dense_ctas CTAs
+// walk their share of the dense items (longest first, snake order), holding
+// 512 TMEM columns; the rest run split-KV warps on the same shared memory.
 //   warp 0      TMA producer: K and V tiles (8 pages, one 128B-swizzled box
 //               per page and operand) into a 2-stage ring, running ahead
 //               across item boundaries; lane i loads page i's id two tiles
@@ -42,6 +41,7 @@
 // never a named barrier), drains its copies and MMAs, frees TMEM and returns.
 #include "kernels.h"
 #include "ptx.cuh"
+#include "split_kv.cuh"
 
 namespace tpa {
 
@@ -57,12 +57,6 @@ __device__ __forceinline__ float fast_exp2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
-}
-
-// Order this thread's generic-proxy global writes before later async-proxy
-// (TMA) reads of the same memory.
-__device__ __forceinline__ void fence_proxy_async_global() {
-  asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
 __device__ __forceinline__ void softmax_bar() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
@@ -115,10 +109,43 @@ __device__ __forceinline__ TileInfo tile_at(const DenseItem& it, int j) {
   return t;
 }
 
-// k-th item of this CTA: snake order over CTAs on a longest-first list.
-__device__ __forceinline__ int item_of(int k) {
-  const int g = static_cast<int>(gridDim.x);
+// k-th item of this dense CTA: snake order over the dense CTAs on a
+// longest-first list.
+__device__ __forceinline__ int item_of(int k, int g) {
   return k * g + ((k & 1) ? g - 1 - static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x));
+}
+
+// Split-KV role of a CTA of the same launch: 8 independent warps, each with
+// a 3-stage TMA page ring in the shared memory the dense role would use.
+constexpr int kSplitWarps = 8;
+constexpr int kSplitStages = 3;
+
+template <int D, int G>
+__device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) {
+  using W = SplitCfg<D, kSplitStages>;
+  static_assert(kSplitWarps * (W::kWarpBytes + kSplitStages * 8) + 16 <= DenseCfg<D>::kOffMisc,
+                "split-KV rings fit in the dense role's shared memory");
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= kSplitWarps) return;
+  uint8_t* ring = smem + warp * W::kWarpBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kSplitWarps * W::kWarpBytes) + warp * kSplitStages;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(
+      smem + kSplitWarps * (W::kWarpBytes + kSplitStages * 8));
+  if (threadIdx.x == 0) *abort_flag = 0;
+  if (lane == 0) {
+    for (int s = 0; s < kSplitStages; ++s) mbar_init(&bars[s], 1);
+    fence_mbar_init();
+  }
+  asm volatile("bar.sync 3, 256;" ::: "memory");
+  if (threadIdx.x == 0) {
+    prefetch_tmap(&p.tmap_k);
+    prefetch_tmap(&p.tmap_v);
+  }
+  SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, p.sitems, p.n_sitems, p.pages,
+              p.squeue, p.status, p.num_pages, p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new,
+              p.k_pool, p.v_pool, p.counters, p.out, p.lse};
+  split_warp_loop<D, G, kSplitStages>(a, ring, bars, abort_flag, lane);
 }
 
 template <int D, int G>
@@ -133,8 +160,13 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
+  if (static_cast<int>(blockIdx.x) >= p.n_dense_ctas) {
+    split_role<D, G>(p, smem);
+    return;
+  }
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int n_ctas = p.n_dense_ctas;
 
   // ---------------------------------------------------------------- setup
   if (threadIdx.x == 0) {
@@ -173,29 +205,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     };
     int gt = 0;  // tiles of this CTA so far (ring position)
     for (int k = 0; pok; ++k) {
-      const int idx = item_of(k);
+      const int idx = item_of(k, n_ctas);
       if (idx >= p.n_items) break;
       const DenseItem item = p.items[idx];
       const int ntiles = item.n_tiles;
-      if (item.app_src >= 0) {
-        // append the step's token to the pool before any key of it is loaded
-        constexpr int U = D / 8;  // 16-byte units of one row
-        const int64_t src = (static_cast<int64_t>(item.app_src) * p.hkv + item.kv_head) * D;
-        const int64_t pg = item.app_dst / kPage;
-        const int64_t dst = ((pg * p.hkv + item.kv_head) * kPage + item.app_dst % kPage) * D;
-        if (pg >= 0 && pg < p.num_pages) {
-          for (int u = lane; u < 2 * U; u += 32) {
-            const bool isv = u >= U;
-            const int uu = isv ? u - U : u;
-            const uint4 v = reinterpret_cast<const uint4*>((isv ? p.v_new : p.k_new) + src)[uu];
-            reinterpret_cast<uint4*>((isv ? p.v_pool : p.k_pool) + dst)[uu] = v;
-          }
-        } else if (lane == 0) {
-          atomicOr(p.status, kStatusBadPage);
-        }
-        fence_proxy_async_global();
-        __syncwarp();
-      }
       auto page_id = [&](int j) -> int32_t {  // raw; validated when used
         if (j >= ntiles) return 0;
         const TileInfo t = tile_at(item, j);
@@ -282,7 +295,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       bool ok = true;
       int gt = 0;
       for (int k = 0; ok; ++k) {
-        const int idx = item_of(k);
+        const int idx = item_of(k, n_ctas);
         if (idx >= p.n_items) break;
         const int ntiles = p.items[idx].n_tiles;
         // Q of this item is written by the softmax warps only after the
@@ -355,7 +368,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     };
     int gt = 0;
     for (int k = 0;; ++k) {
-      const int idx = item_of(k);
+      const int idx = item_of(k, n_ctas);
       if (idx >= p.n_items) break;
       const DenseItem item = p.items[idx];
       const int ntiles = item.n_tiles;
@@ -617,21 +630,20 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 }
 
 template <int D, int G>
-cudaError_t launch_dense_t(const DenseParams& p, int num_sms, cudaStream_t stream) {
-  const int grid = p.n_items < num_sms ? p.n_items : num_sms;
-  dense_kernel<D, G><<<grid, kThreads, DenseCfg<D>::kSmem, stream>>>(p);
+cudaError_t launch_dense_t(const DenseParams& p, int n_split_ctas, cudaStream_t stream) {
+  dense_kernel<D, G><<<p.n_dense_ctas + n_split_ctas, kThreads, DenseCfg<D>::kSmem, stream>>>(p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_dense(const DenseParams& p, int num_sms, int head_dim, int group,
+cudaError_t launch_dense(const DenseParams& p, int n_split_ctas, int head_dim, int group,
                          cudaStream_t stream) {
-  if (p.n_items <= 0) return cudaSuccess;
-  if (head_dim == 128 && group == 4) return launch_dense_t<128, 4>(p, num_sms, stream);
-  if (head_dim == 128 && group == 8) return launch_dense_t<128, 8>(p, num_sms, stream);
-  if (head_dim == 64 && group == 4) return launch_dense_t<64, 4>(p, num_sms, stream);
-  if (head_dim == 64 && group == 8) return launch_dense_t<64, 8>(p, num_sms, stream);
+  if (p.n_dense_ctas + n_split_ctas <= 0) return cudaSuccess;
+  if (head_dim == 128 && group == 4) return launch_dense_t<128, 4>(p, n_split_ctas, stream);
+  if (head_dim == 128 && group == 8) return launch_dense_t<128, 8>(p, n_split_ctas, stream);
+  if (head_dim == 64 && group == 4) return launch_dense_t<64, 4>(p, n_split_ctas, stream);
+  if (head_dim == 64 && group == 8) return launch_dense_t<64, 8>(p, n_split_ctas, stream);
   return cudaErrorInvalidValue;
 }
 

@@ -41,21 +41,26 @@ struct DenseParams {
   const DenseItem* items;
   const DenseTok* toks;
   const int32_t* pages;
-  const __nv_bfloat16* k_new;  // rows appended by items with app_src >= 0
+  const __nv_bfloat16* k_new;  // rows appended by split items with app_src >= 0
   const __nv_bfloat16* v_new;
   __nv_bfloat16* k_pool;
   __nv_bfloat16* v_pool;
   uint32_t* counters;  // zeroed [q rows][hkv] arrival counts; non-null: merge partials in-kernel
   uint32_t* status;
   int64_t num_pages;
-  int n_items;
+  int n_items;       // dense items (128-row tiles)
+  int n_dense_ctas;  // CTAs running dense items; the rest of the grid runs split-KV items
+  const SuffixItem* sitems;
+  int n_sitems;
+  uint32_t* squeue;  // zeroed work counter of the split-KV items
   int hq, hkv;
   float scale_log2;  // log2(e) / sqrt(d)
 };
 
-// Persistent dense tensor-core attention over a list of 128-row query tiles
-// (tcgen05 + TMEM + TMA), one CTA per SM at most.
-cudaError_t launch_dense(const DenseParams& p, int num_sms, int head_dim, int group,
+// One persistent launch, one CTA per SM: the first n_dense_ctas CTAs run the
+// dense tensor-core items (tcgen05 + TMEM + TMA), the others the split-KV
+// items (warp MMA).  Grid = n_dense_ctas + n_split_ctas.
+cudaError_t launch_dense(const DenseParams& p, int n_split_ctas, int head_dim, int group,
                          cudaStream_t stream);
 
 struct SuffixParams {
@@ -72,6 +77,14 @@ struct SuffixParams {
   int n_items;
   int hq, hkv;
   float scale_log2;
+  // in-kernel append and merge (cascade decode); null otherwise
+  const __nv_bfloat16* k_new;
+  const __nv_bfloat16* v_new;
+  __nv_bfloat16* k_pool;
+  __nv_bfloat16* v_pool;
+  uint32_t* counters;
+  __nv_bfloat16* out;
+  float* lse;
 };
 
 // Split-KV paged attention of G query rows per warp (warp-level MMA).

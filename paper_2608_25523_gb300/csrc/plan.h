@@ -44,8 +44,7 @@ struct DenseItem {
   int32_t seg_k0[2];      // first key of the range (multiple of 16)
   int32_t seg_k1[2];      // one past the last key of the range (k1 == k0: empty)
   int32_t seg_causal[2];  // 1: causal mask on this segment
-  int32_t app_src;        // decode: row of k_new/v_new appended before the keys are read (-1: none)
-  int32_t app_dst;        // page * 16 + slot the appended row goes to
+  int32_t pad[2];
 };
 static_assert(sizeof(DenseItem) == 64, "DenseItem layout");
 
@@ -59,9 +58,11 @@ struct SuffixItem {
   int32_t slot_base;  // partial slot of (token, head 0, split 0)
   int32_t n_slots;
   int32_t split;
-  int32_t pad;
+  int32_t app_src;    // decode: row of k_new/v_new appended before the range is read (-1: none)
+  int32_t app_dst;    // page * 16 + slot the appended row goes to
+  int32_t pad[3];
 };
-static_assert(sizeof(SuffixItem) == 32, "SuffixItem layout");
+static_assert(sizeof(SuffixItem) == 48, "SuffixItem layout");
 
 // LSE merge of all partials of one token (every q head).
 struct MergeTok {

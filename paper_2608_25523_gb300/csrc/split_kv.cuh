@@ -1,0 +1,325 @@
+// Split-KV paged attention, one warp per work item: the second level of the
+// decode cascade.
+//
+// Every request adds a private dynamic suffix (plus its decode tokens) to
+// the shared agent prefix (Sec. III, Eq. 2: d_r(t) on top of ell_a), so its
+// suffix keys are read by that request alone.  A work item is the G =
+// Hq/Hkv query rows of one token against one key range of one page run (a
+// request suffix, or in the flat cross-check mode also a prefix); it yields
+// a partial (o, lse).  In the cascade decode the item holding a request's
+// last key first appends the step's token to the pool, and the item that
+// completes the last partial of a (token, kv head) merges all of them by
+// log-sum-exp.
+//
+// Design (memory-bound: ~4 flop per KV byte at G=4):
+//  * each page of one kv head is one TMA box per operand (128-byte swizzle)
+//    landing in a per-warp ring of S stages, so loads run S pages ahead;
+//  * S^T tiles use mma.sync m16n8k16 with the G query rows on the M side
+//    (padded to 16) and the 16 keys of the page on N; P*V reuses the S
+//    accumulators as the A operand (no shared-memory round trip); V comes
+//    through ldmatrix.trans;
+//  * online softmax in base 2 with fp32 accumulators;
+//  * warps pull items from an atomic counter (items sorted longest first).
+#pragma once
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace tpa {
+
+struct SplitArgs {
+  const CUtensorMap* tmap_k;  // kernel-parameter tensor maps of the pools
+  const CUtensorMap* tmap_v;
+  const __nv_bfloat16* q;
+  float* part_o;
+  float* part_lse;
+  const SuffixItem* items;
+  int n_items;
+  const int32_t* pages;
+  uint32_t* queue;
+  uint32_t* status;
+  int64_t num_pages;
+  int hq, hkv;
+  float scale_log2;
+  // cascade decode only (null otherwise): in-kernel append and merge
+  const __nv_bfloat16* k_new;
+  const __nv_bfloat16* v_new;
+  __nv_bfloat16* k_pool;
+  __nv_bfloat16* v_pool;
+  uint32_t* counters;
+  __nv_bfloat16* out;
+  float* lse;
+};
+
+template <int D, int S>
+struct SplitCfg {
+  static constexpr int NCH = D / 64;
+  static constexpr int kPageBytes = NCH * 2048;      // one page of one kv head, K or V
+  static constexpr int kStageBytes = 2 * kPageBytes;
+  static constexpr int kWarpBytes = S * kStageBytes;
+};
+
+namespace split_detail {
+
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+}  // namespace split_detail
+
+// Runs work items until the queue is empty.  `ring` is this warp's S stages,
+// `bars` its S initialised mbarriers (count 1).  Returns false after a
+// timeout (status bit set, in-flight copies drained).
+template <int D, int G, int S>
+__device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bars,
+                                volatile int* abort_flag, int lane) {
+  using namespace split_detail;
+  using C = SplitCfg<D, S>;
+  const int gq = lane >> 2;  // mma group: query row of this lane
+  const int tig = lane & 3;  // thread in group
+  uint32_t it = 0;           // pages consumed by this warp so far (ring position)
+  uint32_t issued = 0;       // pages issued by this warp so far
+  bool failed = false;
+
+  while (!failed) {
+    int idx = 0;
+    if (lane == 0) idx = static_cast<int>(atomicAdd(a.queue, 1u));
+    idx = __shfl_sync(0xffffffffu, idx, 0);
+    if (idx >= a.n_items) break;
+    const SuffixItem item = a.items[idx];
+    const int npg = (item.n_keys + kPage - 1) / kPage;
+
+    if (item.app_src >= 0 && a.k_new) {
+      // append the step's token to the pool before its page is loaded
+      constexpr int U = D / 8;  // 16-byte units of one row
+      const int64_t pg = item.app_dst / kPage;
+      if (pg >= 0 && pg < a.num_pages) {
+        const int64_t src = (static_cast<int64_t>(item.app_src) * a.hkv + item.kv_head) * D;
+        const int64_t dst = ((pg * a.hkv + item.kv_head) * kPage + item.app_dst % kPage) * D;
+        for (int u = lane; u < 2 * U; u += 32) {
+          const bool isv = u >= U;
+          const int uu = isv ? u - U : u;
+          const uint4 v = reinterpret_cast<const uint4*>((isv ? a.v_new : a.k_new) + src)[uu];
+          reinterpret_cast<uint4*>((isv ? a.v_pool : a.k_pool) + dst)[uu] = v;
+        }
+      } else if (lane == 0) {
+        atomicOr(a.status, kStatusBadPage);
+      }
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      __syncwarp();
+    }
+
+    // Query fragments (A operand): rows >= G and the upper 8 rows are zero.
+    uint32_t qa[D / 16][2];
+    {
+      const bool real = gq < G;
+      const __nv_bfloat16* qrow =
+          a.q + (static_cast<int64_t>(item.q_row) * a.hq + item.kv_head * G + (real ? gq : 0)) * D;
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        qa[kk][0] = real ? *reinterpret_cast<const uint32_t*>(qrow + 16 * kk + 2 * tig) : 0u;
+        qa[kk][1] = real ? *reinterpret_cast<const uint32_t*>(qrow + 16 * kk + 8 + 2 * tig) : 0u;
+      }
+    }
+
+    auto issue = [&](int pg) {  // lane 0: TMA page `pg` of the item into ring slot issued % S
+      const int st = static_cast<int>(issued % S);
+      uint8_t* kst = ring + st * C::kStageBytes;
+      uint8_t* vst = kst + C::kPageBytes;
+      int64_t pid = a.pages[item.pages + pg];
+      if (pid < 0 || pid >= a.num_pages) {
+        atomicOr(a.status, kStatusBadPage);
+        pid = 0;
+      }
+      const int z = static_cast<int>(pid * a.hkv + item.kv_head);
+      fence_proxy_async();
+      mbar_arrive_expect_tx(&bars[st], 2 * C::kPageBytes);
+      tma_load_5d(kst, a.tmap_k, &bars[st], 0, 0, 0, 0, z);
+      tma_load_5d(vst, a.tmap_v, &bars[st], 0, 0, 0, 0, z);
+      ++issued;
+    };
+
+    if (lane == 0) {
+      const int pre = npg < S ? npg : S;
+      for (int i = 0; i < pre; ++i) issue(i);
+    }
+    issued = __shfl_sync(0xffffffffu, issued, 0);
+
+    float o[D / 8][4];
+#pragma unroll
+    for (int nt = 0; nt < D / 8; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
+    float m = -INFINITY, l = 0.f;
+
+    for (int pg = 0; pg < npg; ++pg) {
+      const uint32_t cnt = it + pg;
+      const int st = static_cast<int>(cnt % S);
+      if (!__all_sync(0xffffffffu, mbar_wait(&bars[st], (cnt / S) & 1u, abort_flag))) {
+        failed = true;
+        it += pg;  // first page not consumed: pages it .. issued-1 are in flight
+        break;
+      }
+      uint8_t* kst = ring + st * C::kStageBytes;
+      uint8_t* vst = kst + C::kPageBytes;
+      const int valid = item.n_keys - pg * kPage;
+      if (valid < kPage) {
+        // Slots past the end of the run hold stale pool data (possibly not
+        // finite); zero their V rows so 0-weight keys contribute exactly 0.
+        const int nunits = (kPage - valid) * C::NCH * 8;
+        for (int u = lane; u < nunits; u += 32) {
+          const int key = valid + u / (C::NCH * 8);
+          const int cu = u % (C::NCH * 8);
+          *reinterpret_cast<uint4*>(vst + kv_off<C::NCH>(key, cu)) = make_uint4(0, 0, 0, 0);
+        }
+        __syncwarp();
+      }
+      const uint32_t kbase = smem_u32(kst);
+      const uint32_t vbase = smem_u32(vst);
+
+      // S = Q K^T over the page's 16 keys: n-tile 0 = keys 0-7, n-tile 1 = keys 8-15.
+      float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+      {
+        const int key = ((lane >> 4) << 3) + (lane & 7);
+        const int usel = (lane >> 3) & 1;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const int unit = 2 * kk + usel;
+          uint32_t b0, b1, b2, b3;
+          ldmatrix_x4(kbase + kv_off<C::NCH>(key, unit), b0, b1, b2, b3);
+          mma_bf16_16816(s0, qa[kk][0], 0u, qa[kk][1], 0u, b0, b1);
+          mma_bf16_16816(s1, qa[kk][0], 0u, qa[kk][1], 0u, b2, b3);
+        }
+      }
+      const float sc = a.scale_log2;
+      const int k0 = 2 * tig;
+      const float x0 = k0 < valid ? s0[0] * sc : -INFINITY;
+      const float x1 = k0 + 1 < valid ? s0[1] * sc : -INFINITY;
+      const float x2 = k0 + 8 < valid ? s1[0] * sc : -INFINITY;
+      const float x3 = k0 + 9 < valid ? s1[1] * sc : -INFINITY;
+      float mx = fmaxf(fmaxf(x0, x1), fmaxf(x2, x3));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float m_new = fmaxf(m, mx);  // finite: key 0 of every page is valid
+      const float alpha = fast_exp2(m - m_new);
+      const float p0 = fast_exp2(x0 - m_new), p1 = fast_exp2(x1 - m_new);
+      const float p2 = fast_exp2(x2 - m_new), p3 = fast_exp2(x3 - m_new);
+      l = l * alpha + ((p0 + p1) + (p2 + p3));
+      m = m_new;
+#pragma unroll
+      for (int nt = 0; nt < D / 8; ++nt) {
+        o[nt][0] *= alpha;
+        o[nt][1] *= alpha;
+      }
+      const uint32_t pa0 = pack_bf16(p0, p1);
+      const uint32_t pa2 = pack_bf16(p2, p3);
+
+      // O += P V: V rows are keys (k), dims are n; two n-tiles per ldmatrix.x4.trans.
+      {
+        const int mat = lane >> 3;
+        const int key = ((mat & 1) << 3) + (lane & 7);
+#pragma unroll
+        for (int np = 0; np < D / 16; ++np) {
+          const int unit = 2 * np + (mat >> 1);
+          uint32_t b0, b1, b2, b3;
+          ldmatrix_x4_trans(vbase + kv_off<C::NCH>(key, unit), b0, b1, b2, b3);
+          mma_bf16_16816(o[2 * np], pa0, 0u, pa2, 0u, b0, b1);
+          mma_bf16_16816(o[2 * np + 1], pa0, 0u, pa2, 0u, b2, b3);
+        }
+      }
+      __syncwarp();
+      if (lane == 0 && pg + S < npg) issue(pg + S);
+      issued = __shfl_sync(0xffffffffu, issued, 0);
+    }
+    if (failed) break;
+    it += npg;
+
+    l += __shfl_xor_sync(0xffffffffu, l, 1);
+    l += __shfl_xor_sync(0xffffffffu, l, 2);
+    if (gq < G) {
+      const int h = item.kv_head * G + gq;
+      const int64_t slot = item.slot_base + static_cast<int64_t>(h) * item.n_slots + item.split;
+      const float inv = 1.f / l;
+      float* dst = a.part_o + slot * D;
+#pragma unroll
+      for (int nt = 0; nt < D / 8; ++nt)
+        *reinterpret_cast<float2*>(dst + 8 * nt + 2 * tig) =
+            make_float2(o[nt][0] * inv, o[nt][1] * inv);
+      if (tig == 0) a.part_lse[slot] = (m + __log2f(l)) * kLn2;
+    }
+
+    if (a.counters) {
+      // the item completing the last partial of (token, kv head) merges them:
+      // o = sum c_i o_i / sum c_i with c_i = e^(lse_i - M), lse = M + ln sum c_i
+      __threadfence();
+      __syncwarp();
+      uint32_t last = 0;
+      if (lane == 0)
+        last = atomicAdd(a.counters + static_cast<int64_t>(item.q_row) * a.hkv + item.kv_head, 1u) +
+                   1 == static_cast<uint32_t>(item.n_slots);
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
+        __threadfence();
+        constexpr int V = D / 32;  // dims per lane
+        for (int j = 0; j < G; ++j) {
+          const int h = item.kv_head * G + j;
+          const int64_t base = item.slot_base + static_cast<int64_t>(h) * item.n_slots;
+          float mxl = -INFINITY;
+          for (int i = 0; i < item.n_slots; ++i) mxl = fmaxf(mxl, __ldcg(a.part_lse + base + i));
+          float acc[V];
+#pragma unroll
+          for (int c = 0; c < V; ++c) acc[c] = 0.f;
+          float tot = 0.f;
+          for (int i = 0; i < item.n_slots; ++i) {
+            const float w = exp2f((__ldcg(a.part_lse + base + i) - mxl) * kLog2e);
+            tot += w;
+            const float* src = a.part_o + (base + i) * D + lane * V;
+            if constexpr (V == 4) {
+              const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
+              acc[0] += w * v.x;
+              acc[1] += w * v.y;
+              acc[2] += w * v.z;
+              acc[3] += w * v.w;
+            } else {
+              const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
+              acc[0] += w * v.x;
+              acc[1] += w * v.y;
+            }
+          }
+          const float itot = tot > 0.f ? 1.f / tot : 0.f;
+          __nv_bfloat16* dst = a.out + (static_cast<int64_t>(item.q_row) * a.hq + h) * D + lane * V;
+          if constexpr (V == 4) {
+            uint2 pk;
+            pk.x = pack_bf16(acc[0] * itot, acc[1] * itot);
+            pk.y = pack_bf16(acc[2] * itot, acc[3] * itot);
+            *reinterpret_cast<uint2*>(dst) = pk;
+          } else {
+            *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc[0] * itot, acc[1] * itot);
+          }
+          if (lane == 0)
+            a.lse[static_cast<int64_t>(item.q_row) * a.hq + h] =
+                tot > 0.f ? mxl + __log2f(tot) * kLn2 : -INFINITY;
+        }
+      }
+    }
+  }
+
+  if (failed) {
+    if (lane == 0) {
+      atomicOr(a.status, kStatusSuffixTimeout);
+      *abort_flag = 1;
+      // every issued page must land before the CTA exits
+      volatile int never = 0;
+      for (uint32_t c = it; c < issued; ++c) {
+        const int st = static_cast<int>(c % S);
+        (void)mbar_wait(&bars[st], (c / S) & 1u, &never);
+      }
+    }
+    __syncwarp();
+  }
+  return !failed;
+}
+
+}  // namespace tpa

@@ -183,12 +183,11 @@ def test_decode_plan_decomposition(lib):
     ctx.set_option(B.OPT_PREFIX_SPLITS, 4)
     ctx.set_option(B.OPT_SUFFIX_SPLIT_KEYS, 256)
     ctx.decode(list(range(64)), 1, 1, 1, 1, 1)
-    # one persistent tensor-core launch: level 1 = (agent, kv head) x one
-    # 128-row tile (16 tokens x G=4 rows) x 4 key splits; level 2 = per token
-    # and kv head, ceil((len+1)/256) suffix items
-    assert ctx.query(B.Q_LAST_DENSE_ITEMS) == 4 * hkv * 1 * 4 + sum(
-        hkv * math.ceil((l + 1) / 256) for l in lens)
-    assert ctx.query(B.Q_LAST_SUFFIX_ITEMS) == 0
+    # one launch: level 1 (dense CTAs) = (agent, kv head) x one 128-row tile
+    # (16 tokens x G=4 rows) x 4 key splits; level 2 (split-KV CTAs) = per
+    # token and kv head, ceil((len+1)/256) suffix items
+    assert ctx.query(B.Q_LAST_DENSE_ITEMS) == 4 * hkv * 1 * 4
+    assert ctx.query(B.Q_LAST_SUFFIX_ITEMS) == sum(hkv * math.ceil((l + 1) / 256) for l in lens)
     assert ctx.query(B.Q_LAST_LAUNCHES) == 0        # plan-only: nothing launched
     for r in range(64):
         assert ctx.query(B.Q_SUFFIX_LEN, r) == lens[r] + 1
