@@ -1150,13 +1150,14 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       launches = 3;
     } else {
       // one launch, one CTA per SM: dense CTAs for level 1, the rest split-KV;
-      // SMs shared in proportion to estimated time (a dense 128x128 tile
-      // ~1.15 us; split-KV ~35 GB/s of KV per SM)
+      // SMs shared in proportion to estimated time (measured on GB300: a
+      // dense 128x128 tile ~1.6 us when its K/V stream from HBM; split-KV
+      // ~45 GB/s of KV per SM)
       int64_t dense_tiles = 0;
       for (int i = 0; i < nd; ++i) dense_tiles += w.dense[i].n_tiles;
       double split_bytes = 0;
       for (int i = 0; i < ns; ++i) split_bytes += w.suffix[i].n_keys * 4.0 * ctx->d;
-      const double wd = dense_tiles * 1.15, wsplit = split_bytes / 35e3;
+      const double wd = dense_tiles * 1.6, wsplit = split_bytes / 45e3;
       int n_dense = nd == 0 ? 0 : static_cast<int>(std::lround(ctx->num_sms * wd / (wd + wsplit)));
       if (nd > 0) n_dense = std::max(n_dense, 1);
       if (ns > 0) n_dense = std::min(n_dense, ctx->num_sms - 1);

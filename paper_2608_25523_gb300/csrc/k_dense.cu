@@ -195,9 +195,9 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    // Lane i (< 8) owns page i of every tile: it loads that page id two tiles
-    // ahead and issues the page's TMA boxes, so a tile's boxes go out from 8
-    // lanes at once.  Lane 0 posts the expected byte count first.
+    // Lane i (< 8) owns page i of every tile: it loads that page id ahead and
+    // issues the page's TMA boxes, so a tile's boxes go out from 8 lanes at
+    // once.  Lane 0 posts the expected byte count first.
     int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
     bool pok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
@@ -214,7 +214,9 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         const TileInfo t = tile_at(item, j);
         return lane < (t.nvalid + kPage - 1) / kPage ? __ldg(p.pages + t.page_off + lane) : 0;
       };
-      int32_t pid0 = page_id(0), pid1 = page_id(1);
+      // page ids three tiles ahead: tile j+2's (loaded an iteration ago) also
+      // drive an L2 prefetch, so HBM reads run ahead of the 2-stage ring
+      int32_t pid0 = page_id(0), pid1 = page_id(1), pid2 = page_id(2);
       for (int j = 0; j < ntiles; ++j, ++gt) {
         const TileInfo t = tile_at(item, j);
         const int s = gt & 1;
@@ -223,7 +225,16 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         const uint32_t bytes = static_cast<uint32_t>(npg * C::kPageBytes);
         const int32_t pid = pid0;
         pid0 = pid1;
-        pid1 = page_id(j + 2);
+        pid1 = pid2;
+        pid2 = page_id(j + 3);
+        if (j + 2 < ntiles) {
+          const TileInfo t2 = tile_at(item, j + 2);
+          if (lane < (t2.nvalid + kPage - 1) / kPage && pid1 >= 0 && pid1 < p.num_pages) {
+            const int z2 = pid1 * p.hkv + item.kv_head;
+            tma_prefetch_5d(&p.tmap_k, 0, 0, 0, 0, z2);
+            tma_prefetch_5d(&p.tmap_v, 0, 0, 0, 0, z2);
+          }
+        }
         const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
         if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
         const int z = (bad ? 0 : pid) * p.hkv + item.kv_head;
