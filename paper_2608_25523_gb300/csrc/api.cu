@@ -917,6 +917,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
 
   // ---- work decomposition -------------------------------------------------
   int64_t split_keys = 0;  // suffix (and, flat, prefix) key range per item
+  int dense_ctas = 0;      // cascade: CTAs running the stacked prefix tiles
   if (flat) {
     int64_t sum_keys = 0;
     for (int i = 0; i < n; ++i) sum_keys += keys_of(i) + lp_of(i);
@@ -935,18 +936,56 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       split_keys *= 2;
     }
   } else {
-    // Level 1 (dense role): stacked prefix tiles; split each agent's prefix
-    // so the dense items number about the dense CTAs' count or more.
-    int64_t dense_units = 0;
-    for (auto& g : groups)
-      if (ctx->agents[g.agent].len > 0)
-        dense_units += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt);
+    // Level 1 (dense CTAs): stacked prefix tiles, each split into `sp` key
+    // ranges; level 2 (split-KV CTAs): the suffixes.  The split count and the
+    // number of dense CTAs are chosen together so that every dense CTA gets
+    // the same whole number m of (near-equal) items while the split-KV CTAs
+    // finish at about the same time.  Rates measured on GB300: a dense
+    // 128x128 tile ~1.6 us; split-KV ~45 GB/s of KV per SM.
+    constexpr double kTileUs = 1.6, kSplitBytesPerUs = 45e3;
+    double split_bytes = 0;
+    for (int i = 0; i < n; ++i) split_bytes += static_cast<double>(keys_of(i)) * hkv * 4.0 * ctx->d;
+    const double w_split = split_bytes / kSplitBytesPerUs;  // SM-microseconds
+    int64_t ptiles_max = 0;
+    for (auto& g : groups) ptiles_max = std::max<int64_t>(ptiles_max, cdiv(ctx->agents[g.agent].len, kTileKeys));
+    int best_sp = 1, best_d = 0;
+    double best_t = 1e300;
+    if (ptiles_max > 0) {
+      const int sp_lo = ctx->prefix_splits > 0 ? ctx->prefix_splits : 1;
+      const int sp_hi = ctx->prefix_splits > 0 ? ctx->prefix_splits
+                                               : static_cast<int>(std::min<int64_t>(16, ptiles_max));
+      for (int sp = sp_lo; sp <= sp_hi; ++sp) {
+        int64_t items = 0, kmax = 0;
+        for (auto& g : groups) {
+          const int64_t pt = cdiv(ctx->agents[g.agent].len, kTileKeys);
+          if (pt == 0) continue;
+          const int64_t k = cdiv(pt, std::min<int64_t>(sp, pt));
+          items += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) * cdiv(pt, k);
+          kmax = std::max(kmax, k);
+        }
+        for (int m = 1; m <= 8; ++m) {
+          int d = static_cast<int>(cdiv(items, m));
+          if (d > ctx->num_sms - (w_split > 0 ? 1 : 0)) continue;
+          const double t_dense = kTileUs * m * kmax;
+          const double t_split = w_split > 0 ? w_split / (ctx->num_sms - d) : 0.0;
+          const double t = std::max(t_dense, t_split);
+          if (t < best_t) {
+            best_t = t;
+            best_sp = sp;
+            best_d = d;
+          }
+        }
+      }
+      if (best_d == 0) {  // more items than SMs at m <= 8: all but one SM dense
+        best_sp = sp_lo;
+        best_d = ctx->num_sms - (w_split > 0 ? 1 : 0);
+      }
+    }
+    dense_ctas = best_d;
     for (auto& g : groups) {
       const int64_t ptiles = cdiv(ctx->agents[g.agent].len, kTileKeys);
       if (ptiles == 0) continue;
-      int64_t ns = ctx->prefix_splits > 0 ? ctx->prefix_splits
-                                           : cdiv(ctx->num_sms / 4, std::max<int64_t>(1, dense_units));
-      ns = std::min<int64_t>(std::max<int64_t>(ns, 1), ptiles);
+      const int64_t ns = std::min<int64_t>(best_sp, ptiles);
       g.tiles_per_split = static_cast<int32_t>(cdiv(ptiles, ns));
       g.n_split = static_cast<int32_t>(cdiv(ptiles, g.tiles_per_split));
       if (g.n_split >= ctx->max_splits)
@@ -1149,19 +1188,8 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       }
       launches = 3;
     } else {
-      // one launch, one CTA per SM: dense CTAs for level 1, the rest split-KV;
-      // SMs shared in proportion to estimated time (measured on GB300: a
-      // dense 128x128 tile ~1.6 us when its K/V stream from HBM; split-KV
-      // ~45 GB/s of KV per SM)
-      int64_t dense_tiles = 0;
-      for (int i = 0; i < nd; ++i) dense_tiles += w.dense[i].n_tiles;
-      double split_bytes = 0;
-      for (int i = 0; i < ns; ++i) split_bytes += w.suffix[i].n_keys * 4.0 * ctx->d;
-      const double wd = dense_tiles * 1.6, wsplit = split_bytes / 45e3;
-      int n_dense = nd == 0 ? 0 : static_cast<int>(std::lround(ctx->num_sms * wd / (wd + wsplit)));
-      if (nd > 0) n_dense = std::max(n_dense, 1);
-      if (ns > 0) n_dense = std::min(n_dense, ctx->num_sms - 1);
-      n_dense = std::min(n_dense, nd);
+      // one launch, one CTA per SM: dense CTAs for level 1, the rest split-KV
+      const int n_dense = std::min(dense_ctas, nd);
       const int n_split = ns > 0 ? std::min<int>(ctx->num_sms - n_dense,
                                                  static_cast<int>(cdiv(ns, kSplitWarpsPerCta)))
                                  : 0;
