@@ -89,12 +89,13 @@ struct Slot {
 
 // Sizes of one plan: number of records per section.
 struct PlanSizes {
-  int64_t pages = 0, append = 0, dense_tok = 0, dense = 0, suffix = 0, merge = 0, counters = 0;
+  int64_t pages = 0, append = 0, dense_tok = 0, dense = 0, suffix = 0, merge = 0, counters = 0,
+          stok = 0, sint = 0;
 };
 
 struct PlanLayout {
   size_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, off_counters,
-      total;
+      off_stok, off_sint, total;
 };
 
 PlanLayout layout_of(const PlanSizes& s) {
@@ -114,6 +115,10 @@ PlanLayout layout_of(const PlanSizes& s) {
   o = align_up(o + s.merge * sizeof(MergeTok), 64);
   l.off_counters = o;
   o = align_up(o + s.counters * 4, 64);
+  l.off_stok = o;
+  o = align_up(o + s.stok * sizeof(SplitTok), 64);
+  l.off_sint = o;
+  o = align_up(o + s.sint * 4, 64);
   l.total = o;
   return l;
 }
@@ -166,8 +171,12 @@ struct tpa_ctx {
   double k_ms[kKernelKinds] = {};
   int64_t k_n[kKernelKinds] = {};
 
-  // scratch for planning (reused to avoid allocations)
-  std::vector<uint8_t> scratch;
+  // per-call stamps and scratch reused across calls (no heap traffic in steady state)
+  uint64_t stamp = 0;
+  std::vector<uint64_t> req_stamp;    // request id -> stamp of the call that saw it
+  std::vector<uint64_t> agent_stamp;  // agent id -> stamp
+  std::vector<int32_t> agent_group;   // agent id -> group index in the current call
+  std::vector<int32_t> order;         // scratch: token order
 };
 
 namespace {
@@ -212,6 +221,8 @@ PlanSizes plan_capacity(const tpa_config* c) {
   s.suffix = R * H * S;
   s.merge = R;
   s.counters = R * H;
+  s.stok = R;
+  s.sint = 2 * R + 1;
   return s;
 }
 
@@ -323,6 +334,8 @@ struct PlanWriter {
   SuffixItem* suffix;
   MergeTok* merge;
   uint32_t* counters;
+  SplitTok* stok;
+  int32_t* sint;
   PlanWriter(uint8_t* b, const PlanLayout& l) : base(b), lay(l) {
     hdr = reinterpret_cast<PlanHeader*>(b);
     std::memset(hdr, 0, sizeof(PlanHeader));
@@ -333,6 +346,8 @@ struct PlanWriter {
     suffix = reinterpret_cast<SuffixItem*>(b + l.off_suffix);
     merge = reinterpret_cast<MergeTok*>(b + l.off_merge);
     counters = reinterpret_cast<uint32_t*>(b + l.off_counters);
+    stok = reinterpret_cast<SplitTok*>(b + l.off_stok);
+    sint = reinterpret_cast<int32_t*>(b + l.off_sint);
   }
 };
 
@@ -352,10 +367,11 @@ int check_batch(tpa_ctx* ctx, int32_t n, const int32_t* reqs, bool need_resident
       return fail(TPA_ERR_NOT_RESIDENT, "prefix of agent %d (request %d) is not resident",
                   ctx->reqs[r].agent, r);
   }
-  std::vector<int32_t> sorted(reqs, reqs + n);
-  std::sort(sorted.begin(), sorted.end());
-  for (int i = 1; i < n; ++i)
-    if (sorted[i] == sorted[i - 1]) return fail(TPA_ERR_INVALID_ARG, "request %d twice", sorted[i]);
+  const uint64_t st = ++ctx->stamp;
+  for (int i = 0; i < n; ++i) {
+    if (ctx->req_stamp[reqs[i]] == st) return fail(TPA_ERR_INVALID_ARG, "request %d twice", reqs[i]);
+    ctx->req_stamp[reqs[i]] = st;
+  }
   return TPA_OK;
 }
 
@@ -435,6 +451,9 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
   ctx->max_splits = splits_of(cfg);
   ctx->agents.resize(cfg->max_agents);
   ctx->reqs.resize(cfg->max_requests);
+  ctx->req_stamp.assign(cfg->max_requests, 0);
+  ctx->agent_stamp.assign(cfg->max_agents, 0);
+  ctx->agent_group.assign(cfg->max_agents, 0);
   ctx->page_tag.assign(cfg->num_pages, 0);
   ctx->free_pages.resize(cfg->num_pages);
   for (int64_t i = 0; i < cfg->num_pages; ++i) ctx->free_pages[i] = static_cast<int32_t>(i);
@@ -899,17 +918,17 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
   std::vector<AgentGroup> groups;
   std::vector<int32_t> group_of(n);
   {
-    std::unordered_map<int32_t, int> gi;
+    const uint64_t st = ++ctx->stamp;
     for (int i = 0; i < n; ++i) {
       const int32_t a = ctx->reqs[reqs[i]].agent;
-      auto it = gi.find(a);
-      if (it == gi.end()) {
-        gi[a] = static_cast<int>(groups.size());
-        groups.push_back(AgentGroup{a, {i}});
-      } else {
-        groups[it->second].toks.push_back(i);
+      if (ctx->agent_stamp[a] != st) {
+        ctx->agent_stamp[a] = st;
+        ctx->agent_group[a] = static_cast<int32_t>(groups.size());
+        groups.push_back(AgentGroup{a, {}});
+        groups.back().toks.reserve(n);
       }
-      group_of[i] = gi[a];
+      group_of[i] = ctx->agent_group[a];
+      groups[group_of[i]].toks.push_back(i);
     }
   }
   auto keys_of = [&](int i) -> int64_t { return ctx->reqs[reqs[i]].len + 1; };  // with the new token
@@ -1034,7 +1053,8 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     sz.dense_tok = n;
     sz.counters = static_cast<int64_t>(n) * hkv;
     for (auto& g : groups) sz.dense += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) * g.n_split;
-    for (int i = 0; i < n; ++i) sz.suffix += hkv * cdiv(keys_of(i), split_keys);
+    sz.stok = n;
+    sz.sint = 2 * static_cast<int64_t>(n) + 1;
   }
   const PlanLayout lay = layout_of(sz);
   if (lay.total > ctx->plan_cap)
@@ -1065,7 +1085,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     np += static_cast<int32_t>(r.pages.size());
   }
 
-  int32_t nd = 0, ns = 0, nt = 0;
+  int32_t nd = 0, ns = 0, nt = 0, n_full = 0;
   if (flat) {
     write_append_rows(ctx, n, reqs, ones.data(), w.append);
     for (int i = 0; i < n; ++i) w.merge[i] = MergeTok{i, slot_base[i], n_slots[i], 0};
@@ -1115,27 +1135,32 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
           }
       }
     }
-    // level 2: each token's suffix per kv head on the split-KV role; the item
-    // holding the last key appends the step's token first
+    // level 2: one record per token; the split-KV warps derive the items
+    // (full key ranges first, then the tails by decreasing length) and the
+    // item holding a request's last key appends the step's token first
+    int32_t* full_prefix = w.sint;
+    int32_t* tail_order = w.sint + n + 1;
+    full_prefix[0] = 0;
+    std::vector<int32_t>& ord = ctx->order;
+    ord.clear();
     for (int i = 0; i < n; ++i) {
       const Request& r = ctx->reqs[reqs[i]];
       const int64_t keys = keys_of(i);
       const int pos = r.len;  // slot of the new token
-      const int32_t app_dst = r.pages[pos / kPage] * kPage + pos % kPage;
-      int split = groups[group_of[i]].n_split;
-      for (int64_t k0 = 0; k0 < keys; k0 += split_keys, ++split) {
-        const bool last = k0 + split_keys >= keys;
-        for (int h = 0; h < hkv; ++h)
-          w.suffix[ns++] = SuffixItem{i, h, static_cast<int32_t>(suf_off[i] + k0 / kPage),
-                                      static_cast<int32_t>(std::min<int64_t>(split_keys, keys - k0)),
-                                      slot_base[i], n_slots[i], split, last ? i : -1,
-                                      last ? app_dst : 0, {0, 0, 0}};
-      }
+      w.stok[i] = SplitTok{i, suf_off[i], static_cast<int32_t>(keys), slot_base[i], n_slots[i],
+                           groups[group_of[i]].n_split, r.pages[pos / kPage] * kPage + pos % kPage, 0};
+      full_prefix[i + 1] = full_prefix[i] + static_cast<int32_t>(keys / split_keys);
+      if (keys % split_keys) ord.push_back(i);
     }
+    std::sort(ord.begin(), ord.end(), [&](int32_t x, int32_t y) {
+      const int64_t rx = keys_of(x) % split_keys, ry = keys_of(y) % split_keys;
+      return rx != ry ? rx > ry : x < y;
+    });
+    for (size_t t = 0; t < ord.size(); ++t) tail_order[t] = ord[t];
+    n_full = full_prefix[n];
+    ns = hkv * (n_full + static_cast<int32_t>(ord.size()));
     std::stable_sort(w.dense, w.dense + nd,
                      [](const DenseItem& a, const DenseItem& b) { return a.n_tiles > b.n_tiles; });
-    std::stable_sort(w.suffix, w.suffix + ns,
-                     [](const SuffixItem& a, const SuffixItem& b) { return a.n_keys > b.n_keys; });
   }
 
   PlanHeader* hd = w.hdr;
@@ -1195,7 +1220,12 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
                                  : 0;
       DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
       dp.n_dense_ctas = n_dense;
-      dp.sitems = dev_ptr<SuffixItem>(sl, lay.off_suffix);
+      dp.stoks = dev_ptr<SplitTok>(sl, lay.off_stok);
+      dp.full_prefix = dev_ptr<int32_t>(sl, lay.off_sint);
+      dp.tail_order = dev_ptr<int32_t>(sl, lay.off_sint) + n + 1;
+      dp.n_stok = n;
+      dp.n_full = n_full;
+      dp.split_keys = static_cast<int32_t>(split_keys);
       dp.n_sitems = ns;
       dp.squeue = reinterpret_cast<uint32_t*>(sl->dev + offsetof(PlanHeader, queue));
       dp.k_new = static_cast<const __nv_bfloat16*>(k_new);

@@ -142,7 +142,8 @@ __device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) 
     prefetch_tmap(&p.tmap_k);
     prefetch_tmap(&p.tmap_v);
   }
-  SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, p.sitems, p.n_sitems, p.pages,
+  SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, nullptr, p.n_sitems,
+              p.stoks, p.full_prefix, p.tail_order, p.n_stok, p.n_full, p.split_keys, p.pages,
               p.squeue, p.status, p.num_pages, p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new,
               p.k_pool, p.v_pool, p.counters, p.out, p.lse};
   split_warp_loop<D, G, kSplitStages>(a, ring, bars, abort_flag, lane);

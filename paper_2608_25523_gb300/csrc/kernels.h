@@ -50,8 +50,12 @@ struct DenseParams {
   int64_t num_pages;
   int n_items;       // dense items (128-row tiles)
   int n_dense_ctas;  // CTAs running dense items; the rest of the grid runs split-KV items
-  const SuffixItem* sitems;
-  int n_sitems;
+  // split-KV items, derived on the device from per-token records (SplitArgs)
+  const SplitTok* stoks;
+  const int32_t* full_prefix;
+  const int32_t* tail_order;
+  int n_stok, n_full, split_keys;
+  int n_sitems;      // hkv * (n_full + tails)
   uint32_t* squeue;  // zeroed work counter of the split-KV items
   int hq, hkv;
   float scale_log2;  // log2(e) / sqrt(d)

@@ -64,6 +64,20 @@ struct SuffixItem {
 };
 static_assert(sizeof(SuffixItem) == 48, "SuffixItem layout");
 
+// Per-token record of the cascade decode's split-KV level: the suffix of
+// one token's request, cut into key ranges of `split_keys` keys; the work
+// items (token, range, kv head) are derived from these on the device.
+struct SplitTok {
+  int32_t q_row;      // token row (q / out / lse) and row of k_new / v_new
+  int32_t pages;      // page-list offset of the request's suffix page 0
+  int32_t keys;       // suffix keys, the step's token included
+  int32_t slot_base;  // partial slot of (token, head 0, split 0)
+  int32_t n_slots;    // partials per (token, head): prefix splits + suffix ranges
+  int32_t split0;     // split index of the first suffix range (= prefix splits)
+  int32_t app_dst;    // page * 16 + slot of the step's token
+  int32_t pad;
+};
+
 // LSE merge of all partials of one token (every q head).
 struct MergeTok {
   int32_t q_row;

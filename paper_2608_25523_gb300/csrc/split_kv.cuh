@@ -32,8 +32,15 @@ struct SplitArgs {
   const __nv_bfloat16* q;
   float* part_o;
   float* part_lse;
-  const SuffixItem* items;
+  const SuffixItem* items;    // explicit items, or null: derived from toks (below)
   int n_items;
+  // derived items (cascade decode): item idx -> unit idx / hkv, kv head idx % hkv;
+  // units [0, n_full) are full ranges (token found in full_prefix), the rest
+  // are tails in tail_order
+  const SplitTok* toks;
+  const int32_t* full_prefix;  // [n_tok + 1] cumulative full ranges per token
+  const int32_t* tail_order;   // tokens with a tail, longest tail first
+  int n_tok, n_full, split_keys;
   const int32_t* pages;
   uint32_t* queue;
   uint32_t* status;
@@ -69,6 +76,43 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// Work item `idx` (explicit, or derived from the per-token records).
+__device__ __forceinline__ SuffixItem fetch_item(const SplitArgs& a, int idx) {
+  if (a.items) return a.items[idx];
+  const int u = idx / a.hkv;
+  int tok, s, k0, k1;
+  if (u < a.n_full) {
+    int lo = 0, hi = a.n_tok;  // full_prefix[lo] <= u < full_prefix[hi]
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (__ldg(a.full_prefix + mid) <= u) lo = mid;
+      else hi = mid;
+    }
+    tok = lo;
+    s = u - __ldg(a.full_prefix + lo);
+    k0 = s * a.split_keys;
+    k1 = k0 + a.split_keys;
+  } else {
+    tok = __ldg(a.tail_order + (u - a.n_full));
+    const int keys = __ldg(&a.toks[tok].keys);
+    s = keys / a.split_keys;
+    k0 = s * a.split_keys;
+    k1 = keys;
+  }
+  const SplitTok t = a.toks[tok];
+  SuffixItem it;
+  it.q_row = t.q_row;
+  it.kv_head = idx % a.hkv;
+  it.pages = t.pages + k0 / kPage;
+  it.n_keys = k1 - k0;
+  it.slot_base = t.slot_base;
+  it.n_slots = t.n_slots;
+  it.split = t.split0 + s;
+  it.app_src = k1 == t.keys ? t.q_row : -1;
+  it.app_dst = t.app_dst;
+  return it;
+}
+
 }  // namespace split_detail
 
 // Runs work items until the queue is empty.  `ring` is this warp's S stages,
@@ -90,7 +134,7 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
     if (lane == 0) idx = static_cast<int>(atomicAdd(a.queue, 1u));
     idx = __shfl_sync(0xffffffffu, idx, 0);
     if (idx >= a.n_items) break;
-    const SuffixItem item = a.items[idx];
+    const SuffixItem item = fetch_item(a, idx);
     const int npg = (item.n_keys + kPage - 1) / kPage;
 
     if (item.app_src >= 0 && a.k_new) {
