@@ -89,13 +89,13 @@ struct Slot {
 
 // Sizes of one plan: number of records per section.
 struct PlanSizes {
-  int64_t pages = 0, append = 0, dense_tok = 0, dense = 0, suffix = 0, merge = 0, counters = 0,
-          stok = 0, sint = 0;
+  int64_t pages = 0, append = 0, dense_tok = 0, dense = 0, suffix = 0, merge = 0, stok = 0,
+          sint = 0;
 };
 
 struct PlanLayout {
-  size_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, off_counters,
-      off_stok, off_sint, total;
+  size_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, off_stok,
+      off_sint, total;
 };
 
 PlanLayout layout_of(const PlanSizes& s) {
@@ -113,8 +113,6 @@ PlanLayout layout_of(const PlanSizes& s) {
   o = align_up(o + s.suffix * sizeof(SuffixItem), 64);
   l.off_merge = o;
   o = align_up(o + s.merge * sizeof(MergeTok), 64);
-  l.off_counters = o;
-  o = align_up(o + s.counters * 4, 64);
   l.off_stok = o;
   o = align_up(o + s.stok * sizeof(SplitTok), 64);
   l.off_sint = o;
@@ -220,7 +218,6 @@ PlanSizes plan_capacity(const tpa_config* c) {
   s.dense = H * std::max((cdiv(R, tpt) + A) * S + R * S, cdiv(T, tpt) + R);
   s.suffix = R * H * S;
   s.merge = R;
-  s.counters = R * H;
   s.stok = R;
   s.sint = 2 * R + 1;
   return s;
@@ -333,7 +330,6 @@ struct PlanWriter {
   DenseItem* dense;
   SuffixItem* suffix;
   MergeTok* merge;
-  uint32_t* counters;
   SplitTok* stok;
   int32_t* sint;
   PlanWriter(uint8_t* b, const PlanLayout& l) : base(b), lay(l) {
@@ -345,7 +341,6 @@ struct PlanWriter {
     dense = reinterpret_cast<DenseItem*>(b + l.off_dense);
     suffix = reinterpret_cast<SuffixItem*>(b + l.off_suffix);
     merge = reinterpret_cast<MergeTok*>(b + l.off_merge);
-    counters = reinterpret_cast<uint32_t*>(b + l.off_counters);
     stok = reinterpret_cast<SplitTok*>(b + l.off_stok);
     sint = reinterpret_cast<int32_t*>(b + l.off_sint);
   }
@@ -1051,7 +1046,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       sz.suffix += hkv * (cdiv(keys_of(i), split_keys) + cdiv(lp_of(i), split_keys));
   } else {
     sz.dense_tok = n;
-    sz.counters = static_cast<int64_t>(n) * hkv;
+    sz.merge = n;
     for (auto& g : groups) sz.dense += static_cast<int64_t>(hkv) * cdiv(g.toks.size(), tpt) * g.n_split;
     sz.stok = n;
     sz.sint = 2 * static_cast<int64_t>(n) + 1;
@@ -1104,7 +1099,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     std::stable_sort(w.suffix, w.suffix + ns,
                      [](const SuffixItem& a, const SuffixItem& b) { return a.n_keys > b.n_keys; });
   } else {
-    std::memset(w.counters, 0, static_cast<size_t>(n) * hkv * 4);
+    for (int i = 0; i < n; ++i) w.merge[i] = MergeTok{i, slot_base[i], n_slots[i], 0};
     // level 1: stacked prefix tiles of each agent
     for (auto& g : groups) {
       if (g.n_split == 0) continue;
@@ -1169,8 +1164,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
   hd->n_dense_tok = nt;
   hd->n_dense = nd;
   hd->n_suffix = ns;
-  hd->n_merge = flat ? n : 0;
-  hd->n_counters = flat ? 0 : n * hkv;
+  hd->n_merge = n;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   chain_begin(ctx, s);
@@ -1209,7 +1203,8 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       {
         KernelTimer kt(ctx, K_MERGE, s);
         CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
-                              static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, s));
+                              static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, ctx->num_sms,
+                              true, s));
       }
       launches = 3;
     } else {
@@ -1230,10 +1225,18 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       dp.squeue = reinterpret_cast<uint32_t*>(sl->dev + offsetof(PlanHeader, queue));
       dp.k_new = static_cast<const __nv_bfloat16*>(k_new);
       dp.v_new = static_cast<const __nv_bfloat16*>(v_new);
-      dp.counters = reinterpret_cast<uint32_t*>(sl->dev + lay.off_counters);
-      KernelTimer kt(ctx, K_DENSE, s);
-      CUDA_TRY(launch_dense(dp, n_split, ctx->d, G, s));
-      launches = 1;
+      {
+        KernelTimer kt(ctx, K_DENSE, s);
+        CUDA_TRY(launch_dense(dp, n_split, ctx->d, G, s));
+      }
+      {
+        // a programmatic dependent: resident before the main kernel ends
+        KernelTimer kt(ctx, K_MERGE, s);
+        CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
+                              static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, ctx->num_sms,
+                              true, s));
+      }
+      launches = 2;
     }
   }
   for (int i = 0; i < n; ++i) {

@@ -11,9 +11,8 @@
 //    cores once per tile instead of once per request;
 //  * decode, level 2 runs in the same launch on the other CTAs (split_kv.cuh:
 //    one warp per request suffix range, which also appends the step's token);
-//  * decode partials are merged exactly by log-sum-exp inside the kernel:
-//    the item (of either role) that completes the last partial of a (token,
-//    kv head) merges them (arrival counters in the plan);
+//    both levels write fp32 partials (o, lse) that the merge kernel, launched
+//    as a programmatic dependent of this one, combines exactly;
 //  * chunked causal prefill (Sec. VI cites chunked prefill): a tile of one
 //    request's chunk attends to the whole prefix and causally to the
 //    request's own suffix, writing final outputs directly.
@@ -29,13 +28,15 @@
 //               PV is ready first (QK may run two tiles ahead of PV):
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
 //                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
-//   warps 2..9  two per TMEM lane quarter: warp 2+q+4h owns rows 32q..32q+31
-//               and key half h.  Per item: load their part of Q, then per
-//               tile read S, take the full-row max (both warps of a pair, so
-//               their running max agrees without synchronising), write P for
-//               their key half, rescale O in TMEM only when the max grew by
-//               more than 2^8 (otherwise the stale max stays the reference,
-//               which is exact: it is only a stabiliser); then the epilogue.
+//   warps 2..9  warp w owns TMEM lane quarter w % 4 (rows 32(w%4)..+31) and
+//               key half (w-2)/4.  Per tile: read S, take the full-row max
+//               (both warps of a pair, so their running max agrees without
+//               synchronising), write P for their key half, rescale O in
+//               TMEM only when the max grew by more than 2^8 (otherwise the
+//               stale max stays the reference, which is exact: it is only a
+//               stabiliser); then the item's epilogue.  The next item's Q
+//               rows are copied in (cp.async) as soon as the current item's
+//               last QK has completed, so its first QKs overlap the epilogue.
 // Every mbarrier wait is bounded.  On a timeout the CTA records a status bit
 // and every role still walks the same item/tile sequence (skipping the work,
 // never a named barrier), drains its copies and MMAs, frees TMEM and returns.
@@ -48,7 +49,6 @@ namespace tpa {
 namespace {
 
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 constexpr int kThreads = 320;               // producer, MMA, 8 softmax warps
 constexpr int kSoftmax = 256;
@@ -78,8 +78,7 @@ struct DenseCfg {
   static constexpr int kOffBar = kOffV + kStages * kKVBytes;
   static constexpr int kNumBars = 16;
   static constexpr int kOffL = kOffBar + kNumBars * 8;   // partial row sums [2][128]
-  static constexpr int kOffFlag = kOffL + 2 * 128 * 4;   // merge flags per token [32]
-  static constexpr int kOffMisc = kOffFlag + 32 * 4;
+  static constexpr int kOffMisc = kOffL + 2 * 128 * 4;
   static constexpr int kSmem = 1024 + kOffMisc + 64;
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
@@ -145,7 +144,7 @@ __device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) 
   SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, nullptr, p.n_sitems,
               p.stoks, p.full_prefix, p.tail_order, p.n_stok, p.n_full, p.split_keys, p.pages,
               p.squeue, p.status, p.num_pages, p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new,
-              p.k_pool, p.v_pool, p.counters, p.out, p.lse};
+              p.k_pool, p.v_pool};
   split_warp_loop<D, G, kSplitStages>(a, ring, bars, abort_flag, lane);
 }
 
@@ -157,10 +156,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kOffBar);
   float* lpart = reinterpret_cast<float*>(smem + C::kOffL);
-  int* mflag = reinterpret_cast<int*>(smem + C::kOffFlag);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
+  pdl_trigger();  // the merge kernel after a decode may become resident now
   if (static_cast<int>(blockIdx.x) >= p.n_dense_ctas) {
     split_role<D, G>(p, smem);
     return;
@@ -268,6 +267,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         if (vph_last[s] >= 0) (void)mbar_wait(&bars[B_VFULL + s], vph_last[s], &never);
       }
     }
+    __syncwarp();  // the warp reaches the teardown barrier converged
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -310,8 +310,9 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         const int idx = item_of(k, n_ctas);
         if (idx >= p.n_items) break;
         const int ntiles = p.items[idx].n_tiles;
-        // Q of this item is written by the softmax warps only after the
-        // previous item's last PV completed (so Q and O are free again)
+        // Q of this item is copied in by the softmax warps once the previous
+        // item's last QK has completed; O is overwritten only by this item's
+        // first PV, whose P comes after they have read the previous O out
         if (!mbar_wait(&bars[B_QFULL], k & 1, abort_flag)) { ok = false; break; }
         // Issue whichever is ready first: QK of the next tile (K landed, its S
         // buffer released by the softmax two tiles back) or PV of the oldest
@@ -356,6 +357,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       volatile int never = 0;
       (void)mbar_wait(&bars[B_DRAIN], 0, &never);
     }
+    // lanes 1..31 wait here for the issuing lane: an aligned CTA barrier
+    // must see the warp converged, or it may release before every TMEM
+    // reader is done
+    __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax
     // Every softmax thread walks the same items and tiles even after a
@@ -378,39 +383,73 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       *abort_flag = 1;  // let the other roles stop waiting too
       return false;
     };
+    // This thread's half of its Q row for an item (zero for padding rows),
+    // copied straight into the swizzled Q tile.  The next item's copy starts
+    // as soon as this item's last QK has completed, and Q_FULL is signalled
+    // before this item's epilogue, so the next item's first QKs overlap it.
+    auto load_q = [&](const DenseTok& t, int kv_head, bool valid) {
+      constexpr int U = D / 16;
+      const int head = kv_head * G + row % G;
+      const __nv_bfloat16* src =
+          p.q + (valid ? (static_cast<int64_t>(t.q_row) * p.hq + head) * D + half * (D / 2) : 0);
+      uint8_t* qs = smem + C::kOffQ;
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int gu = half * U + u;
+        cp_async_16(qs + (gu >> 3) * C::kChunk + swz128(row, gu & 7), src + 8 * u, valid ? 16u : 0u);
+      }
+      cp_async_commit();
+    };
+    auto q_ready = [&]() {
+      cp_async_wait_all();
+      fence_proxy_async();
+      mbar_arrive(&bars[B_QFULL]);
+    };
+    constexpr DenseTok kNoTok = {0, 0x7fffffff, 0, 0};
+    // descriptors of the item after the current one, loaded an item ahead
+    DenseTok dt_next = kNoTok;
+    int kv_next = 0;
+    bool valid_next = false;
+    {
+      const int idx0 = item_of(0, n_ctas);
+      if (idx0 < p.n_items) {
+        kv_next = p.items[idx0].kv_head;
+        valid_next = tok < p.items[idx0].n_tok;
+        if (valid_next) dt_next = p.toks[p.items[idx0].tok_base + tok];
+        load_q(dt_next, kv_next, valid_next);
+        q_ready();
+      }
+    }
     int gt = 0;
     for (int k = 0;; ++k) {
       const int idx = item_of(k, n_ctas);
       if (idx >= p.n_items) break;
       const DenseItem item = p.items[idx];
       const int ntiles = item.n_tiles;
-      const bool row_valid = tok < item.n_tok;
-      DenseTok dt = {0, 0x7fffffff, 0, 0};
-      if (row_valid) dt = p.toks[item.tok_base + tok];
+      const bool row_valid = valid_next;
+      const DenseTok dt = dt_next;
       const int head = item.kv_head * G + row % G;
-      {
-        // this thread's half of its Q row (zero for padding rows)
-        constexpr int U = D / 16;
-        uint8_t* qs = smem + C::kOffQ;
-        const uint4* src = reinterpret_cast<const uint4*>(
-            p.q + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D) + half * U;
-        uint4 v[U];
-#pragma unroll
-        for (int u = 0; u < U; ++u) v[u] = row_valid ? src[u] : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const int gu = half * U + u;
-          *reinterpret_cast<uint4*>(qs + (gu >> 3) * C::kChunk + swz128(row, gu & 7)) = v[u];
-        }
-        fence_proxy_async();
-        mbar_arrive(&bars[B_QFULL]);
+      const int idx_n = item_of(k + 1, n_ctas);
+      const bool has_next = idx_n < p.n_items;
+      dt_next = kNoTok;
+      valid_next = false;
+      if (has_next) {
+        kv_next = p.items[idx_n].kv_head;
+        valid_next = tok < p.items[idx_n].n_tok;
+        if (valid_next) dt_next = p.toks[p.items[idx_n].tok_base + tok];
       }
+      bool q_issued = false;
       float m_run = -INFINITY, l_run = 0.f;
       for (int j = 0; j < ntiles && ok; ++j) {
         const TileInfo t = tile_at(item, j);
         const int g = gt + j;
         const int s = g & 1;
         if (!wait_all(&bars[B_SFULL + s], (g >> 1) & 1)) { ok = false; break; }
+        if (j == ntiles - 1 && has_next) {
+          // the item's last QK has completed: its Q tile is free
+          load_q(dt_next, kv_next, valid_next);
+          q_issued = true;
+        }
         tc_fence_after();
         const uint32_t scol = tmem + lane_base + (s ? C::kColS1 : C::kColS0);
         float x[64], y[64];
@@ -525,6 +564,11 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         mbar_arrive(&bars[B_PFULL]);
       }
 
+      if (has_next) {
+        if (!q_issued) load_q(dt_next, kv_next, valid_next);
+        q_ready();
+      }
+
       // ---------------------------------------------------------- epilogue
       lpart[half * 128 + row] = l_run;
       softmax_bar();
@@ -569,63 +613,9 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           else p.lse[static_cast<int64_t>(dt.q_row) * p.hq + head] = lse;
         }
       }
-      if (item.out_mode == 0 && p.counters) {
-        // the item that completes the last partial of a (token, kv head)
-        // merges all of them: o = sum c_i o_i / sum c_i, c_i = e^(lse_i - M)
-        __threadfence();
-        softmax_bar();
-        if (half == 0 && row % G == 0) {
-          int last = 0;
-          if (row_valid && ok) {
-            const uint32_t prev = atomicAdd(
-                p.counters + static_cast<int64_t>(dt.q_row) * p.hkv + item.kv_head, 1u);
-            last = prev + 1 == static_cast<uint32_t>(dt.n_slots);
-          }
-          mflag[tok] = last;
-        }
-        softmax_bar();
-        if (row_valid && mflag[tok]) {
-          __threadfence();
-          const int64_t base = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots;
-          float mxl = -INFINITY;
-          for (int i = 0; i < dt.n_slots; ++i) mxl = fmaxf(mxl, __ldcg(p.part_lse + base + i));
-          float macc[D / 2];
-#pragma unroll
-          for (int c = 0; c < D / 2; ++c) macc[c] = 0.f;
-          float tot = 0.f;
-          for (int i = 0; i < dt.n_slots; ++i) {
-            const float w = exp2f((__ldcg(p.part_lse + base + i) - mxl) * kLog2e);
-            tot += w;
-            const float4* src =
-                reinterpret_cast<const float4*>(p.part_o + (base + i) * D + half * (D / 2));
-#pragma unroll
-            for (int c = 0; c < D / 8; ++c) {
-              const float4 v = __ldcg(src + c);
-              macc[4 * c] += w * v.x;
-              macc[4 * c + 1] += w * v.y;
-              macc[4 * c + 2] += w * v.z;
-              macc[4 * c + 3] += w * v.w;
-            }
-          }
-          const float itot = tot > 0.f ? 1.f / tot : 0.f;
-          uint4* dst = reinterpret_cast<uint4*>(
-              p.out + (static_cast<int64_t>(dt.q_row) * p.hq + head) * D + half * (D / 2));
-#pragma unroll
-          for (int c = 0; c < D / 16; ++c) {
-            uint4 v;
-            v.x = pack_bf16(macc[8 * c + 0] * itot, macc[8 * c + 1] * itot);
-            v.y = pack_bf16(macc[8 * c + 2] * itot, macc[8 * c + 3] * itot);
-            v.z = pack_bf16(macc[8 * c + 4] * itot, macc[8 * c + 5] * itot);
-            v.w = pack_bf16(macc[8 * c + 6] * itot, macc[8 * c + 7] * itot);
-            dst[c] = v;
-          }
-          if (half == 0)
-            p.lse[static_cast<int64_t>(dt.q_row) * p.hq + head] =
-                tot > 0.f ? mxl + __log2f(tot) * kLn2 : -INFINITY;
-        }
-      }
       gt += ntiles;
     }
+    cp_async_wait_all();
     if (!ok) {
       *abort_flag = 1;
       atomicOr(p.status, kStatusDenseTimeout);

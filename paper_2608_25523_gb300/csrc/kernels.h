@@ -45,7 +45,6 @@ struct DenseParams {
   const __nv_bfloat16* v_new;
   __nv_bfloat16* k_pool;
   __nv_bfloat16* v_pool;
-  uint32_t* counters;  // zeroed [q rows][hkv] arrival counts; non-null: merge partials in-kernel
   uint32_t* status;
   int64_t num_pages;
   int n_items;       // dense items (128-row tiles)
@@ -81,14 +80,11 @@ struct SuffixParams {
   int n_items;
   int hq, hkv;
   float scale_log2;
-  // in-kernel append and merge (cascade decode); null otherwise
+  // in-kernel append of the step's token (cascade decode); null otherwise
   const __nv_bfloat16* k_new;
   const __nv_bfloat16* v_new;
   __nv_bfloat16* k_pool;
   __nv_bfloat16* v_pool;
-  uint32_t* counters;
-  __nv_bfloat16* out;
-  float* lse;
 };
 
 // Split-KV paged attention of G query rows per warp (warp-level MMA).
@@ -96,9 +92,12 @@ cudaError_t launch_suffix(const SuffixParams& p, int num_sms, int head_dim, int 
                           cudaStream_t stream);
 
 // Exact LSE merge of each token's partials into bf16 out and fp32 lse.
+// dependent = true launches it as a programmatic dependent of the kernel
+// before it on the stream (which triggers early): its CTAs become resident
+// while that kernel still runs and start merging the moment it completes.
 cudaError_t launch_merge(const MergeTok* toks, int n_tok, const float* part_o,
                          const float* part_lse, __nv_bfloat16* out, float* lse, int hq, int d,
-                         cudaStream_t stream);
+                         int num_sms, bool dependent, cudaStream_t stream);
 
 // Raise dynamic shared-memory limits of the kernels (once per device).
 cudaError_t init_kernels();

@@ -88,8 +88,8 @@ struct MergeTok {
 
 // Header of an uploaded plan blob; offsets in bytes from the blob start.
 struct PlanHeader {
-  int32_t n_pages, n_append, n_dense_tok, n_dense, n_suffix, n_merge, n_counters;
-  int32_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge, off_counters;
+  int32_t n_pages, n_append, n_dense_tok, n_dense, n_suffix, n_merge;
+  int32_t off_pages, off_append, off_dense_tok, off_dense, off_suffix, off_merge;
   uint32_t queue[4];  // zero on upload: atomic work counters of persistent kernels
 };
 

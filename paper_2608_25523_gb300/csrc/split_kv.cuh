@@ -47,14 +47,11 @@ struct SplitArgs {
   int64_t num_pages;
   int hq, hkv;
   float scale_log2;
-  // cascade decode only (null otherwise): in-kernel append and merge
+  // cascade decode only (null otherwise): in-kernel append of the step's token
   const __nv_bfloat16* k_new;
   const __nv_bfloat16* v_new;
   __nv_bfloat16* k_pool;
   __nv_bfloat16* v_pool;
-  uint32_t* counters;
-  __nv_bfloat16* out;
-  float* lse;
 };
 
 template <int D, int S>
@@ -68,7 +65,6 @@ struct SplitCfg {
 namespace split_detail {
 
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
@@ -292,61 +288,6 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
         *reinterpret_cast<float2*>(dst + 8 * nt + 2 * tig) =
             make_float2(o[nt][0] * inv, o[nt][1] * inv);
       if (tig == 0) a.part_lse[slot] = (m + __log2f(l)) * kLn2;
-    }
-
-    if (a.counters) {
-      // the item completing the last partial of (token, kv head) merges them:
-      // o = sum c_i o_i / sum c_i with c_i = e^(lse_i - M), lse = M + ln sum c_i
-      __threadfence();
-      __syncwarp();
-      uint32_t last = 0;
-      if (lane == 0)
-        last = atomicAdd(a.counters + static_cast<int64_t>(item.q_row) * a.hkv + item.kv_head, 1u) +
-                   1 == static_cast<uint32_t>(item.n_slots);
-      last = __shfl_sync(0xffffffffu, last, 0);
-      if (last) {
-        __threadfence();
-        constexpr int V = D / 32;  // dims per lane
-        for (int j = 0; j < G; ++j) {
-          const int h = item.kv_head * G + j;
-          const int64_t base = item.slot_base + static_cast<int64_t>(h) * item.n_slots;
-          float mxl = -INFINITY;
-          for (int i = 0; i < item.n_slots; ++i) mxl = fmaxf(mxl, __ldcg(a.part_lse + base + i));
-          float acc[V];
-#pragma unroll
-          for (int c = 0; c < V; ++c) acc[c] = 0.f;
-          float tot = 0.f;
-          for (int i = 0; i < item.n_slots; ++i) {
-            const float w = exp2f((__ldcg(a.part_lse + base + i) - mxl) * kLog2e);
-            tot += w;
-            const float* src = a.part_o + (base + i) * D + lane * V;
-            if constexpr (V == 4) {
-              const float4 v = __ldcg(reinterpret_cast<const float4*>(src));
-              acc[0] += w * v.x;
-              acc[1] += w * v.y;
-              acc[2] += w * v.z;
-              acc[3] += w * v.w;
-            } else {
-              const float2 v = __ldcg(reinterpret_cast<const float2*>(src));
-              acc[0] += w * v.x;
-              acc[1] += w * v.y;
-            }
-          }
-          const float itot = tot > 0.f ? 1.f / tot : 0.f;
-          __nv_bfloat16* dst = a.out + (static_cast<int64_t>(item.q_row) * a.hq + h) * D + lane * V;
-          if constexpr (V == 4) {
-            uint2 pk;
-            pk.x = pack_bf16(acc[0] * itot, acc[1] * itot);
-            pk.y = pack_bf16(acc[2] * itot, acc[3] * itot);
-            *reinterpret_cast<uint2*>(dst) = pk;
-          } else {
-            *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc[0] * itot, acc[1] * itot);
-          }
-          if (lane == 0)
-            a.lse[static_cast<int64_t>(item.q_row) * a.hq + h] =
-                tot > 0.f ? mxl + __log2f(tot) * kLn2 : -INFINITY;
-        }
-      }
     }
   }
 
