@@ -195,6 +195,30 @@ TPA_API int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, cons
 TPA_API int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q,
                const void* k_new, const void* v_new, void* out, float* lse, void* stream);
 
+/* tpa_decode with its split partial results in a fixed device array
+ * instead of the context's workspace.  The paper has no counterpart: this
+ * is an allocation-free variant of the decode step for callers that want
+ * its scratch to come from static device memory.
+ *   Arguments, layouts and results are those of tpa_decode, and the outputs
+ *   are bit-identical to it.  The scratch is a 256-byte aligned file-scope
+ *   __device__ array of 16 MiB per device inside this library: fp32 partial
+ *   outputs [slots][d] followed by their fp32 LSEs, so it holds
+ *   slots = (16 MiB - 256) / (4 (d + 1)) partials (32510 at d = 128).  Its
+ *   address is looked up once per device (with that device current) and
+ *   cached; the call allocates no device or pinned memory.
+ *   Nothing in the array has to start at zero: every partial a call reads
+ *   is written earlier in the same call.
+ *   All calls of this entry point on one device share the array: calls
+ *   whose kernels overlap in time (other streams, other contexts, other
+ *   threads) race on it and their outputs are undefined.  Order them on
+ *   one stream, or use tpa_decode.
+ * Errors: those of tpa_decode; CAPACITY (message names the limit) when the
+ * step needs more partial slots than the array holds; CUDA when the array's
+ * address cannot be looked up. */
+TPA_API int tpa_decode_static_scratch(tpa_ctx* ctx, int32_t n, const int32_t* reqs,
+                                      const void* q, const void* k_new, const void* v_new,
+                                      void* out, float* lse, void* stream);
+
 /* Copy a prefix (is_request = 0) or a request suffix (is_request = 1) out of
  * its pages into contiguous bf16 [len][Hkv][d] arrays `k_out`, `v_out`
  * (device or pinned host memory).  Errors: INVALID_ARG, STATE, NOT_RESIDENT. */

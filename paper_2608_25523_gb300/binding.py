@@ -71,6 +71,8 @@ _SIGS = {
                                   c_void_p, c_void_p, c_void_p, c_void_p]),
     "tpa_decode": (c_int, [c_void_p, c_int32, _I32P, c_void_p, c_void_p, c_void_p, c_void_p,
                            c_void_p, c_void_p]),
+    "tpa_decode_static_scratch": (c_int, [c_void_p, c_int32, _I32P, c_void_p, c_void_p,
+                                          c_void_p, c_void_p, c_void_p, c_void_p]),
     "tpa_gather": (c_int, [c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
     "tpa_query": (c_int, [c_void_p, c_int32, c_int32, POINTER(c_int64)]),
     "tpa_set_option": (c_int, [c_void_p, c_int32, c_int64]),
@@ -214,6 +216,12 @@ class Context:
         return self._check(self.lib.tpa_decode(self.handle, len(reqs), _i32(reqs), _ptr(q),
                                                _ptr(k_new), _ptr(v_new), _ptr(out), _ptr(lse),
                                                _stream(stream)))
+
+    def decode_static_scratch(self, reqs, q, k_new, v_new, out, lse, stream=None):
+        """decode() with its split partials in the library's static device array."""
+        return self._check(self.lib.tpa_decode_static_scratch(
+            self.handle, len(reqs), _i32(reqs), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out),
+            _ptr(lse), _stream(stream)))
 
     def gather(self, ident, is_request, k_out, v_out, stream=None):
         return self._check(self.lib.tpa_gather(self.handle, ident, 1 if is_request else 0,

@@ -1382,6 +1382,39 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   return finish_call(ctx, sl, s, true);
 }
 
+int tpa_decode_static_scratch(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q,
+                              const void* k_new, const void* v_new, void* out, float* lse,
+                              void* stream) {
+  if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");
+  // [slots][d] fp32 partial outputs, then [slots] fp32 partial LSEs
+  const size_t bytes = static_scratch_bytes();
+  const int64_t slots = static_cast<int64_t>((bytes - kAlign) / ((ctx->d + 1) * sizeof(float)));
+  void* base = nullptr;
+  if (!ctx->plan_only) {
+    const cudaError_t e = static_scratch(ctx->device, &base);
+    if (e != cudaSuccess)
+      return fail(TPA_ERR_CUDA, "static scratch address: %s", cudaGetErrorString(e));
+  }
+  float* const saved_o = ctx->part_o;
+  float* const saved_lse = ctx->part_lse;
+  const int64_t saved_slots = ctx->part_slots;
+  ctx->part_o = static_cast<float*>(base);
+  ctx->part_lse = base ? reinterpret_cast<float*>(static_cast<uint8_t*>(base) +
+                                                  align_up(slots * ctx->d * sizeof(float), kAlign))
+                       : nullptr;
+  ctx->part_slots = slots;
+  int rc = tpa_decode(ctx, n, reqs, q, k_new, v_new, out, lse, stream);
+  ctx->part_o = saved_o;
+  ctx->part_lse = saved_lse;
+  ctx->part_slots = saved_slots;
+  if (rc == TPA_ERR_CAPACITY && g_err == "partial slots exhausted")
+    rc = fail(TPA_ERR_CAPACITY,
+              "decode needs more split partials than the %zu-byte static scratch holds "
+              "(%lld slots of head_dim %d)",
+              bytes, static_cast<long long>(slots), ctx->d);
+  return rc;
+}
+
 int tpa_gather(tpa_ctx* ctx, int32_t id, int32_t is_request, void* k_out, void* v_out,
                void* stream) {
   if (!ctx) return fail(TPA_ERR_INVALID_ARG, "null context");

@@ -102,4 +102,10 @@ cudaError_t launch_merge(const MergeTok* toks, int n_tok, const float* part_o,
 // Raise dynamic shared-memory limits of the kernels (once per device).
 cudaError_t init_kernels();
 
+// The 256-byte aligned static device array behind tpa_decode_static_scratch:
+// its size, and its address on `device` (looked up once per device with that
+// device current; no allocation).
+size_t static_scratch_bytes();
+cudaError_t static_scratch(int device, void** ptr);
+
 }  // namespace tpa
