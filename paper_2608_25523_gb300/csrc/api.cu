@@ -84,6 +84,7 @@ struct Slot {
   uint8_t* host = nullptr;   // pinned staging
   uint8_t* dev = nullptr;    // device copy (workspace)
   cudaEvent_t done = nullptr;
+  cudaStream_t stream = nullptr;  // stream `done` was recorded on
   uint64_t seq = 0;          // call that used the slot last (0: never)
 };
 
@@ -228,6 +229,9 @@ void wait_for_seq(tpa_ctx* ctx, uint64_t seq, cudaStream_t s) {
   if (seq == 0 || ctx->plan_only) return;
   for (auto& sl : ctx->ring) {
     if (sl.seq == seq) {
+      // work already queued on `s` is ordered before what follows on `s`; an
+      // event wait would only stall the queue until that call has drained
+      if (sl.stream == s) return;
       if (cudaEventQuery(sl.done) == cudaErrorNotReady) cudaStreamWaitEvent(s, sl.done, 0);
       else (void)cudaGetLastError();
       return;
@@ -390,6 +394,7 @@ int finish_call(tpa_ctx* ctx, Slot* sl, cudaStream_t s, bool chain) {
   }
   if (ctx->plan_only) return TPA_OK;
   CUDA_TRY(cudaEventRecord(sl->done, s));
+  sl->stream = s;
   return TPA_OK;
 }
 
@@ -954,9 +959,11 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     // ranges; level 2 (split-KV CTAs): the suffixes.  The split count and the
     // number of dense CTAs are chosen together so that every dense CTA gets
     // the same whole number m of (near-equal) items while the split-KV CTAs
-    // finish at about the same time.  Rates measured on GB300: a dense
-    // 128x128 tile ~1.6 us; split-KV ~45 GB/s of KV per SM.
-    constexpr double kTileUs = 1.6, kSplitBytesPerUs = 45e3;
+    // finish at about the same time.  Rates measured on GB300 with both
+    // roles streaming: a dense 128x128 tile ~2 us, plus ~2 us per item (the
+    // next item's Q is loaded once the previous item's last QK is done);
+    // split-KV ~50 GB/s of KV per SM.  Ties go to fewer splits.
+    constexpr double kTileUs = 2.0, kItemUs = 2.0, kSplitBytesPerUs = 50e3;
     double split_bytes = 0;
     for (int i = 0; i < n; ++i) split_bytes += static_cast<double>(keys_of(i)) * hkv * 4.0 * ctx->d;
     const double w_split = split_bytes / kSplitBytesPerUs;  // SM-microseconds
@@ -980,7 +987,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
         for (int m = 1; m <= 8; ++m) {
           int d = static_cast<int>(cdiv(items, m));
           if (d > ctx->num_sms - (w_split > 0 ? 1 : 0)) continue;
-          const double t_dense = kTileUs * m * kmax;
+          const double t_dense = (kTileUs * kmax + kItemUs) * m;
           const double t_split = w_split > 0 ? w_split / (ctx->num_sms - d) : 0.0;
           const double t = std::max(t_dense, t_split);
           if (t < best_t) {

@@ -203,20 +203,36 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
       return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
     };
+    auto page_id = [&](const DenseItem& it, int j) -> int32_t {  // raw; validated when used
+      if (j >= it.n_tiles) return 0;
+      const TileInfo t = tile_at(it, j);
+      return lane < (t.nvalid + kPage - 1) / kPage ? __ldg(p.pages + t.page_off + lane) : 0;
+    };
+    // The current item and its first three tiles' page ids.  The next item's
+    // are loaded while the current one streams (the descriptor after tile 0
+    // is issued, the page ids after tile 1), so item boundaries add no load
+    // latency to the TMA stream.
+    DenseItem item{};
+    int32_t f0 = 0, f1 = 0, f2 = 0;
+    if (item_of(0, n_ctas) < p.n_items) {
+      item = p.items[item_of(0, n_ctas)];
+      f0 = page_id(item, 0);
+      f1 = page_id(item, 1);
+      f2 = page_id(item, 2);
+    }
     int gt = 0;  // tiles of this CTA so far (ring position)
     for (int k = 0; pok; ++k) {
       const int idx = item_of(k, n_ctas);
       if (idx >= p.n_items) break;
-      const DenseItem item = p.items[idx];
       const int ntiles = item.n_tiles;
-      auto page_id = [&](int j) -> int32_t {  // raw; validated when used
-        if (j >= ntiles) return 0;
-        const TileInfo t = tile_at(item, j);
-        return lane < (t.nvalid + kPage - 1) / kPage ? __ldg(p.pages + t.page_off + lane) : 0;
-      };
+      const int idx_n = item_of(k + 1, n_ctas);
+      const bool has_next = idx_n < p.n_items;
+      DenseItem nitem{};
+      int32_t n0 = 0, n1 = 0, n2 = 0;
+      bool next_ready = false;
       // page ids three tiles ahead: tile j+2's (loaded an iteration ago) also
       // drive an L2 prefetch, so HBM reads run ahead of the 2-stage ring
-      int32_t pid0 = page_id(0), pid1 = page_id(1), pid2 = page_id(2);
+      int32_t pid0 = f0, pid1 = f1, pid2 = f2;
       for (int j = 0; j < ntiles; ++j, ++gt) {
         const TileInfo t = tile_at(item, j);
         const int s = gt & 1;
@@ -226,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         const int32_t pid = pid0;
         pid0 = pid1;
         pid1 = pid2;
-        pid2 = page_id(j + 3);
+        pid2 = page_id(item, j + 3);
         if (j + 2 < ntiles) {
           const TileInfo t2 = tile_at(item, j + 2);
           if (lane < (t2.nvalid + kPage - 1) / kPage && pid1 >= 0 && pid1 < p.num_pages) {
@@ -252,7 +268,24 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           tma_load_5d(smem + C::kOffV + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_v,
                       &bars[B_VFULL + s], 0, 0, 0, 0, z);
         vph_last[s] = static_cast<int>(ph);
+        if (has_next && j == 0) nitem = p.items[idx_n];
+        if (has_next && j == 1) {
+          n0 = page_id(nitem, 0);
+          n1 = page_id(nitem, 1);
+          n2 = page_id(nitem, 2);
+          next_ready = true;
+        }
       }
+      if (has_next && !next_ready) {
+        if (ntiles == 0) nitem = p.items[idx_n];
+        n0 = page_id(nitem, 0);
+        n1 = page_id(nitem, 1);
+        n2 = page_id(nitem, 2);
+      }
+      item = nitem;
+      f0 = n0;
+      f1 = n1;
+      f2 = n2;
     }
     if (!pok && lane == 0) {
       *abort_flag = 1;
