@@ -146,8 +146,9 @@ struct tpa_ctx {
   float* part_o = nullptr;
   float* part_lse = nullptr;
   int64_t part_slots = 0;
-  size_t plan_cap = 0;
+  size_t plan_cap = 0;               // bytes of a plan slot; its upload flag follows it
   Slot ring[kRingSlots];
+  cudaStream_t copy_stream = nullptr;  // decode plans are uploaded here, ahead of the kernels
   int ring_pos = 0;
   uint64_t seq = 0;
   uint64_t chain_seq = 0;            // last chain (ordered) call
@@ -386,6 +387,24 @@ int upload(tpa_ctx* ctx, Slot* sl, size_t bytes, cudaStream_t s) {
   return TPA_OK;
 }
 
+// Upload a plan on the context's copy stream, followed by the call's
+// sequence number into the slot's flag word: the kernel reading the plan
+// waits (bounded) for that flag, so the call's own stream carries only
+// kernels and the next step's kernel can be a programmatic dependent of the
+// previous one.  The slot is reused only after its call's done event, which
+// follows a kernel that saw the flag, so the copies have completed by then.
+int upload_ahead(tpa_ctx* ctx, Slot* sl, size_t bytes, const unsigned long long** flag) {
+  *flag = nullptr;
+  if (ctx->plan_only) return TPA_OK;
+  uint64_t* fh = reinterpret_cast<uint64_t*>(sl->host + ctx->plan_cap);
+  *fh = ctx->seq;
+  CUDA_TRY(cudaMemcpyAsync(sl->dev, sl->host, bytes, cudaMemcpyHostToDevice, ctx->copy_stream));
+  CUDA_TRY(cudaMemcpyAsync(sl->dev + ctx->plan_cap, fh, sizeof(uint64_t), cudaMemcpyHostToDevice,
+                           ctx->copy_stream));
+  *flag = reinterpret_cast<const unsigned long long*>(sl->dev + ctx->plan_cap);
+  return TPA_OK;
+}
+
 int finish_call(tpa_ctx* ctx, Slot* sl, cudaStream_t s, bool chain) {
   sl->seq = ctx->seq;
   if (chain) {
@@ -411,7 +430,7 @@ size_t tpa_workspace_size(const tpa_config* cfg) {
   const PlanLayout lay = layout_of(plan_capacity(cfg));
   const int64_t slots = max_batch_requests(cfg) * cfg->num_q_heads * splits_of(cfg);
   size_t total = kAlign;                                     // status word
-  total += kRingSlots * align_up(lay.total, kAlign);         // plan ring
+  total += kRingSlots * (align_up(lay.total, kAlign) + kAlign);  // plan ring (+ upload flags)
   total += align_up(slots * cfg->head_dim * sizeof(float), kAlign);
   total += align_up(slots * sizeof(float), kAlign);
   return total;
@@ -527,21 +546,27 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
   size_t off = kAlign;
   for (auto& s : ctx->ring) {
     s.dev = ws + off;
-    off += ctx->plan_cap;
+    off += ctx->plan_cap + kAlign;
   }
   ctx->part_o = reinterpret_cast<float*>(ws + off);
   off += align_up(ctx->part_slots * ctx->d * sizeof(float), kAlign);
   ctx->part_lse = reinterpret_cast<float*>(ws + off);
 
   for (auto& s : ctx->ring) {
-    if ((e = cudaHostAlloc(reinterpret_cast<void**>(&s.host), ctx->plan_cap, cudaHostAllocDefault)) !=
-        cudaSuccess)
+    if ((e = cudaHostAlloc(reinterpret_cast<void**>(&s.host), ctx->plan_cap + kAlign,
+                           cudaHostAllocDefault)) != cudaSuccess)
       return cleanup(fail(TPA_ERR_CUDA, "pinned staging: %s", cudaGetErrorString(e)));
     if ((e = cudaEventCreateWithFlags(&s.done, cudaEventDisableTiming)) != cudaSuccess)
       return cleanup(fail(TPA_ERR_CUDA, "event: %s", cudaGetErrorString(e)));
   }
-  if ((e = cudaMemsetAsync(ctx->status, 0, sizeof(uint32_t), 0)) != cudaSuccess ||
-      (e = cudaStreamSynchronize(0)) != cudaSuccess)
+  if ((e = cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking)) != cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "copy stream: %s", cudaGetErrorString(e)));
+  if ((e = cudaMemsetAsync(ctx->status, 0, sizeof(uint32_t), 0)) != cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "status init: %s", cudaGetErrorString(e)));
+  for (auto& s : ctx->ring)
+    if ((e = cudaMemsetAsync(s.dev + ctx->plan_cap, 0, sizeof(uint64_t), 0)) != cudaSuccess)
+      return cleanup(fail(TPA_ERR_CUDA, "flag init: %s", cudaGetErrorString(e)));
+  if ((e = cudaStreamSynchronize(0)) != cudaSuccess)
     return cleanup(fail(TPA_ERR_CUDA, "status init: %s", cudaGetErrorString(e)));
   (void)rc;
   *out = ctx;
@@ -562,6 +587,10 @@ int tpa_destroy(tpa_ctx* ctx) {
     }
     resolve_timing(ctx);
     for (cudaEvent_t e : ctx->ev_free) cudaEventDestroy(e);
+    if (ctx->copy_stream) {
+      cudaStreamSynchronize(ctx->copy_stream);
+      cudaStreamDestroy(ctx->copy_stream);
+    }
   }
   delete ctx;
   return TPA_OK;
@@ -1177,7 +1206,9 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
   chain_begin(ctx, s);
   wait_for_seq(ctx, tag, s);
   for (auto& g : groups) wait_for_seq(ctx, ctx->agents[g.agent].ready_seq, s);
-  if ((rc = upload(ctx, sl, lay.total, s))) return rc;
+  const unsigned long long* plan_flag = nullptr;
+  if ((rc = flat ? upload(ctx, sl, lay.total, s) : upload_ahead(ctx, sl, lay.total, &plan_flag)))
+    return rc;
 
   int launches = 0;
   if (!ctx->plan_only) {
@@ -1233,8 +1264,11 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       dp.k_new = static_cast<const __nv_bfloat16*>(k_new);
       dp.v_new = static_cast<const __nv_bfloat16*>(v_new);
       {
-        KernelTimer kt(ctx, K_DENSE, s);
-        CUDA_TRY(launch_dense(dp, n_split, ctx->d, G, s));
+          KernelTimer kt(ctx, K_DENSE, s);
+        dp.plan_flag = plan_flag;
+        dp.plan_seq = ctx->seq;
+        // a programmatic dependent of the previous step's merge on this stream
+        CUDA_TRY(launch_dense(dp, n_split, ctx->d, G, true, s));
       }
       {
         // a programmatic dependent: resident before the main kernel ends
@@ -1375,7 +1409,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
     DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
     dp.n_dense_ctas = std::min(nd, ctx->num_sms);
     KernelTimer kt(ctx, K_DENSE, s);
-    CUDA_TRY(launch_dense(dp, 0, ctx->d, G, s));
+    CUDA_TRY(launch_dense(dp, 0, ctx->d, G, false, s));
   }
   for (int i = 0; i < n; ++i) {
     Request& r = ctx->reqs[reqs[i]];

@@ -160,6 +160,15 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
   pdl_trigger();  // the merge kernel after a decode may become resident now
+  if (p.plan_flag) {
+    // the plan came on another stream: wait for its flag (bounded)
+    const int got = threadIdx.x == 0 ? wait_flag64(p.plan_flag, p.plan_seq) : 1;
+    if (!__syncthreads_and(got)) {
+      if (threadIdx.x == 0) atomicOr(p.status, kStatusPlanTimeout);
+      return;
+    }
+  }
+  pdl_wait();  // the kernel before this one (if a programmatic dependent) has completed
   if (static_cast<int>(blockIdx.x) >= p.n_dense_ctas) {
     split_role<D, G>(p, smem);
     return;
@@ -665,20 +674,30 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 }
 
 template <int D, int G>
-cudaError_t launch_dense_t(const DenseParams& p, int n_split_ctas, cudaStream_t stream) {
-  dense_kernel<D, G><<<p.n_dense_ctas + n_split_ctas, kThreads, DenseCfg<D>::kSmem, stream>>>(p);
-  return cudaGetLastError();
+cudaError_t launch_dense_t(const DenseParams& p, int n_split_ctas, bool dependent,
+                           cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(p.n_dense_ctas + n_split_ctas));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = DenseCfg<D>::kSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = dependent ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, dense_kernel<D, G>, p);
 }
 
 }  // namespace
 
 cudaError_t launch_dense(const DenseParams& p, int n_split_ctas, int head_dim, int group,
-                         cudaStream_t stream) {
+                         bool dependent, cudaStream_t stream) {
   if (p.n_dense_ctas + n_split_ctas <= 0) return cudaSuccess;
-  if (head_dim == 128 && group == 4) return launch_dense_t<128, 4>(p, n_split_ctas, stream);
-  if (head_dim == 128 && group == 8) return launch_dense_t<128, 8>(p, n_split_ctas, stream);
-  if (head_dim == 64 && group == 4) return launch_dense_t<64, 4>(p, n_split_ctas, stream);
-  if (head_dim == 64 && group == 8) return launch_dense_t<64, 8>(p, n_split_ctas, stream);
+  if (head_dim == 128 && group == 4) return launch_dense_t<128, 4>(p, n_split_ctas, dependent, stream);
+  if (head_dim == 128 && group == 8) return launch_dense_t<128, 8>(p, n_split_ctas, dependent, stream);
+  if (head_dim == 64 && group == 4) return launch_dense_t<64, 4>(p, n_split_ctas, dependent, stream);
+  if (head_dim == 64 && group == 8) return launch_dense_t<64, 8>(p, n_split_ctas, dependent, stream);
   return cudaErrorInvalidValue;
 }
 

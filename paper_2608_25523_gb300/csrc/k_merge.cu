@@ -27,7 +27,8 @@ __global__ void __launch_bounds__(kMergeThreads)
     merge_kernel(const MergeTok* __restrict__ toks, int n_tok, const float* __restrict__ part_o,
                  const float* __restrict__ part_lse, __nv_bfloat16* __restrict__ out,
                  float* __restrict__ lse_out, int hq) {
-  pdl_wait();  // no-op unless launched as a dependent
+  pdl_trigger();  // the next step's main kernel may become resident now
+  pdl_wait();     // no-op unless launched as a dependent
   constexpr int LPI = D / 4;     // lanes per (token, head)
   constexpr int IPW = 32 / LPI;  // (token, head) pairs per warp and pass
   const int lane = threadIdx.x & 31;

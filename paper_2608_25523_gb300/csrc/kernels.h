@@ -58,13 +58,20 @@ struct DenseParams {
   uint32_t* squeue;  // zeroed work counter of the split-KV items
   int hq, hkv;
   float scale_log2;  // log2(e) / sqrt(d)
+  // Non-null: the plan was uploaded on another stream, followed by this
+  // 8-byte flag; every CTA waits (bounded) until it reads plan_seq there.
+  const unsigned long long* plan_flag;
+  unsigned long long plan_seq;
 };
 
 // One persistent launch, one CTA per SM: the first n_dense_ctas CTAs run the
 // dense tensor-core items (tcgen05 + TMEM + TMA), the others the split-KV
-// items (warp MMA).  Grid = n_dense_ctas + n_split_ctas.
+// items (warp MMA).  Grid = n_dense_ctas + n_split_ctas.  dependent = true
+// launches it as a programmatic dependent of the kernel before it on the
+// stream: its CTAs may start while that kernel finishes and wait for it in
+// griddepcontrol.wait before touching any memory it could use.
 cudaError_t launch_dense(const DenseParams& p, int n_split_ctas, int head_dim, int group,
-                         cudaStream_t stream);
+                         bool dependent, cudaStream_t stream);
 
 struct SuffixParams {
   CUtensorMap tmap_k;

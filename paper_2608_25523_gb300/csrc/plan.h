@@ -13,6 +13,7 @@ constexpr int kTileKeys = 128;     // keys per dense tile (8 pages)
 constexpr uint32_t kStatusDenseTimeout = 1u;
 constexpr uint32_t kStatusSuffixTimeout = 2u;
 constexpr uint32_t kStatusBadPage = 4u;
+constexpr uint32_t kStatusPlanTimeout = 8u;  // a plan upload never arrived
 
 // One token row of a KV write: row `src` of the source K/V arrays goes to
 // slot `slot` of page `page`.

@@ -28,6 +28,20 @@ __device__ __forceinline__ void pdl_trigger() {
 }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// Wait until the 64-bit word at f (written by a copy on another stream)
+// equals want; false after kWaitLimitNs.  Acquire: later loads see what the
+// copies before the flag wrote.
+__device__ __forceinline__ bool wait_flag64(const unsigned long long* f, unsigned long long want) {
+  const unsigned long long t0 = global_ns();
+  for (;;) {
+    unsigned long long v;
+    asm volatile("ld.acquire.sys.global.u64 %0, [%1];" : "=l"(v) : "l"(f) : "memory");
+    if (v == want) return true;
+    if (global_ns() - t0 > kWaitLimitNs) return false;
+    __nanosleep(128);
+  }
+}
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
