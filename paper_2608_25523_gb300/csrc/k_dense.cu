@@ -22,7 +22,7 @@
 // 512 TMEM columns; the rest run split-KV warps on the same shared memory.
 //   warp 0      TMA producer: K and V tiles (8 pages, one 128B-swizzled box
 //               per page and operand) into a 2-stage ring, running ahead
-//               across item boundaries; lane i loads page i's id two tiles
+//               across item boundaries; lane i loads page i's id three tiles
 //               ahead and issues that page's boxes
 //   warp 1      TMEM owner; one lane issues tcgen05.mma, whichever of QK /
 //               PV is ready first (QK may run two tiles ahead of PV):
@@ -73,10 +73,10 @@ struct DenseCfg {
   static constexpr int kStages = 2;
   static constexpr int kOffQ = 0;
   static constexpr int kOffP = kOffQ + kQBytes;
-  static constexpr int kOffK = kOffP + kPBytes;
+  static constexpr int kOffK = kOffP + 2 * kPBytes;  // P is double-buffered
   static constexpr int kOffV = kOffK + kStages * kKVBytes;
   static constexpr int kOffBar = kOffV + kStages * kKVBytes;
-  static constexpr int kNumBars = 16;
+  static constexpr int kNumBars = 18;
   static constexpr int kOffL = kOffBar + kNumBars * 8;   // partial row sums [2][128]
   static constexpr int kOffMisc = kOffL + 2 * 128 * 4;
   static constexpr int kSmem = 1024 + kOffMisc + 64;
@@ -86,7 +86,7 @@ struct DenseCfg {
 
 // barrier slots
 enum { B_KFULL = 0, B_KEMPTY = 2, B_VFULL = 4, B_VEMPTY = 6, B_SFULL = 8, B_SFREE = 10,
-       B_PFULL = 12, B_OFULL = 13, B_QFULL = 14, B_DRAIN = 15 };
+       B_PFULL = 12, B_PVDONE = 14, B_QFULL = 16, B_DRAIN = 17 };
 
 struct TileInfo {
   int key0;     // first key of the tile within its segment
@@ -188,8 +188,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       mbar_init(&bars[B_SFULL + i], 1);
       mbar_init(&bars[B_SFREE + i], kSoftmax);
     }
-    mbar_init(&bars[B_PFULL], kSoftmax);
-    mbar_init(&bars[B_OFULL], 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars[B_PFULL + i], kSoftmax);
+      mbar_init(&bars[B_PVDONE + i], 1);
+    }
     mbar_init(&bars[B_QFULL], kSoftmax);
     mbar_init(&bars[B_DRAIN], 1);
     fence_mbar_init();
@@ -239,8 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       DenseItem nitem{};
       int32_t n0 = 0, n1 = 0, n2 = 0;
       bool next_ready = false;
-      // page ids three tiles ahead: tile j+2's (loaded an iteration ago) also
-      // drive an L2 prefetch, so HBM reads run ahead of the 2-stage ring
+      // page ids loaded three tiles ahead
       int32_t pid0 = f0, pid1 = f1, pid2 = f2;
       for (int j = 0; j < ntiles; ++j, ++gt) {
         const TileInfo t = tile_at(item, j);
@@ -252,14 +253,6 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         pid0 = pid1;
         pid1 = pid2;
         pid2 = page_id(item, j + 3);
-        if (j + 2 < ntiles) {
-          const TileInfo t2 = tile_at(item, j + 2);
-          if (lane < (t2.nvalid + kPage - 1) / kPage && pid1 >= 0 && pid1 < p.num_pages) {
-            const int z2 = pid1 * p.hkv + item.kv_head;
-            tma_prefetch_5d(&p.tmap_k, 0, 0, 0, 0, z2);
-            tma_prefetch_5d(&p.tmap_v, 0, 0, 0, 0, z2);
-          }
-        }
         const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
         if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
         const int z = (bad ? 0 : pid) * p.hkv + item.kv_head;
@@ -339,11 +332,12 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         const uint32_t vb = vbase0 + s * C::kKVBytes;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t a = umma_sdesc(pbase + (kk >> 2) * C::kChunk + (kk & 3) * 32, 16, 1024);
+          const uint64_t a = umma_sdesc(pbase + (g & 1) * C::kPBytes + (kk >> 2) * C::kChunk +
+                                            (kk & 3) * 32, 16, 1024);
           const uint64_t b = umma_sdesc(vb + kk * C::kPageBytes, 1024, C::kGroup);
           umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (!first || kk > 0) ? 1u : 0u);
         }
-        umma_commit(&bars[B_OFULL]);
+        umma_commit(&bars[B_PVDONE + (g & 1)]);
         umma_commit(&bars[B_VEMPTY + s]);
       };
       bool ok = true;
@@ -375,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           }
           if (np < nq) {
             const int g = gt + np;
-            if (mbar_test(&bars[B_PFULL], g & 1) &&
+            if (mbar_test(&bars[B_PFULL + (g & 1)], (g >> 1) & 1) &&
                 mbar_test(&bars[B_VFULL + (g & 1)], (g >> 1) & 1)) {
               issue_pv(g, np == 0);
               ++np;
@@ -551,12 +545,14 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           }
         const float rsum = ((sacc[0] + sacc[1]) + (sacc[2] + sacc[3])) +
                            ((sacc[4] + sacc[5]) + (sacc[6] + sacc[7]));
-        if (j > 0) {
-          if (!wait_all(&bars[B_OFULL], (g - 1) & 1)) { ok = false; break; }
+        // P buffer g % 2 was last read by PV(g - 2)
+        if (g >= 2 && !wait_all(&bars[B_PVDONE + (g & 1)], ((g >> 1) & 1) ^ 1u)) { ok = false; break; }
+        // rescale this half of the O row when the reference max moved (with real
+        // content), after PV(g - 1) has finished accumulating into it
+        if (j > 0 && __any_sync(0xffffffffu, grow && m_run > -INFINITY)) {
+          if (!wait_all(&bars[B_PVDONE + ((g - 1) & 1)], ((g - 1) >> 1) & 1)) { ok = false; break; }
           tc_fence_after();
-          // rescale this half of the O row when the reference max moved (with real content)
-          const bool need = grow && m_run > -INFINITY;
-          if (__any_sync(0xffffffffu, need)) {
+          {
 #pragma unroll 1
             for (int c = 0; c < D / 64; ++c) {
               float o[32];
@@ -599,11 +595,11 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           v.y = pack_bf16(x[8 * u + 2], x[8 * u + 3]);
           v.z = pack_bf16(x[8 * u + 4], x[8 * u + 5]);
           v.w = pack_bf16(x[8 * u + 6], x[8 * u + 7]);
-          *reinterpret_cast<uint4*>(ps + half * C::kChunk + swz128(row, u)) = v;
+          *reinterpret_cast<uint4*>(ps + (g & 1) * C::kPBytes + half * C::kChunk + swz128(row, u)) = v;
         }
         fence_proxy_async();
         tc_fence_before();
-        mbar_arrive(&bars[B_PFULL]);
+        mbar_arrive(&bars[B_PFULL + (g & 1)]);
       }
 
       if (has_next) {
@@ -615,7 +611,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       lpart[half * 128 + row] = l_run;
       softmax_bar();
       const float l_tot = lpart[row] + lpart[128 + row];
-      if (!wait_all(&bars[B_OFULL], (gt + ntiles - 1) & 1)) ok = false;
+      if (ntiles > 0) {
+        const int gl = gt + ntiles - 1;  // the item's last PV
+        if (!wait_all(&bars[B_PVDONE + (gl & 1)], (gl >> 1) & 1)) ok = false;
+      }
       const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
       const float lse = l_tot > 0.f ? (m_run + __log2f(l_tot)) * kLn2 : -INFINITY;
       const int64_t slot = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
