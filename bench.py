@@ -588,6 +588,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed"],
+                    help="run just one of the extra workloads (1 GPU) and print its result")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     rank = int(os.environ.get("RANK", 0))
@@ -597,6 +599,18 @@ def main():
         res = run_reference(args, rank, world)
         if res is not None:
             print(json.dumps(res))
+        return
+    if args.only:
+        import torch
+        from paper_2608_25523_gb300.build import build
+        build()
+        dev = torch.device("cuda", 0)
+        torch.cuda.set_device(dev)
+        hbm_peak, tf_peak, _, peak_src = peaks()
+        fn = {"prefill": lambda: bench_prefill(args, dev, tf_peak, peak_src),
+              "decode_70b": lambda: bench_70b(args, dev, hbm_peak, peak_src),
+              "mixed": lambda: bench_mixed(args, dev)}[args.only]
+        print(json.dumps({"only": args.only, "result": fn()}))
         return
     if world > 1:
         import torch

@@ -141,6 +141,7 @@ struct tpa_ctx {
   int device = 0;
   int num_sms = 148;
   CUtensorMap tmap_k{}, tmap_v{};
+  CUtensorMap* run_maps = nullptr;  // device copy (workspace) of the per-kv-head page-run views
   PoolGeom pool{};
   uint32_t* status = nullptr;
   float* part_o = nullptr;
@@ -430,6 +431,7 @@ size_t tpa_workspace_size(const tpa_config* cfg) {
   const PlanLayout lay = layout_of(plan_capacity(cfg));
   const int64_t slots = max_batch_requests(cfg) * cfg->num_q_heads * splits_of(cfg);
   size_t total = kAlign;                                     // status word
+  total += align_up(2 * static_cast<size_t>(cfg->num_kv_heads) * sizeof(CUtensorMap), kAlign);
   total += kRingSlots * (align_up(lay.total, kAlign) + kAlign);  // plan ring (+ upload flags)
   total += align_up(slots * cfg->head_dim * sizeof(float), kAlign);
   total += align_up(slots * sizeof(float), kAlign);
@@ -538,12 +540,34 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cleanup(fail(TPA_ERR_CUDA, "cuTensorMapEncodeTiled: %d", (int)r));
   }
+  // per-kv-head views for runs of consecutive pages: the kv head is in the
+  // base address and the last dimension steps over pages
+  std::vector<CUtensorMap> runs(2 * static_cast<size_t>(ctx->hkv));
+  {
+    const cuuint64_t rdims[5] = {64, 8, nch, 2, static_cast<cuuint64_t>(cfg->num_pages)};
+    const cuuint64_t rstrides[4] = {row, 128, 8 * row,
+                                    static_cast<cuuint64_t>(ctx->hkv) * kPage * row};
+    const cuuint32_t rbox[5] = {64, 8, static_cast<cuuint32_t>(nch), 2, 8};
+    for (int w = 0; w < 2; ++w)
+      for (int h = 0; h < ctx->hkv; ++h) {
+        void* base = static_cast<uint8_t*>(w ? cfg->v_pool : cfg->k_pool) +
+                     static_cast<size_t>(h) * kPage * row;
+        CUresult r = encode(&runs[w * ctx->hkv + h], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, base,
+                            rdims, rstrides, rbox, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS)
+          return cleanup(fail(TPA_ERR_CUDA, "cuTensorMapEncodeTiled (runs): %d", (int)r));
+      }
+  }
   ctx->pool = PoolGeom{cfg->k_pool, cfg->v_pool, cfg->num_pages, ctx->hkv, ctx->d};
 
   // workspace carve-up
   uint8_t* ws = static_cast<uint8_t*>(cfg->workspace);
   ctx->status = reinterpret_cast<uint32_t*>(ws);
   size_t off = kAlign;
+  ctx->run_maps = reinterpret_cast<CUtensorMap*>(ws + off);
+  off += align_up(runs.size() * sizeof(CUtensorMap), kAlign);
   for (auto& s : ctx->ring) {
     s.dev = ws + off;
     off += ctx->plan_cap + kAlign;
@@ -559,6 +583,9 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
     if ((e = cudaEventCreateWithFlags(&s.done, cudaEventDisableTiming)) != cudaSuccess)
       return cleanup(fail(TPA_ERR_CUDA, "event: %s", cudaGetErrorString(e)));
   }
+  if ((e = cudaMemcpy(ctx->run_maps, runs.data(), runs.size() * sizeof(CUtensorMap),
+                      cudaMemcpyHostToDevice)) != cudaSuccess)
+    return cleanup(fail(TPA_ERR_CUDA, "tensor maps: %s", cudaGetErrorString(e)));
   if ((e = cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking)) != cudaSuccess)
     return cleanup(fail(TPA_ERR_CUDA, "copy stream: %s", cudaGetErrorString(e)));
   if ((e = cudaMemsetAsync(ctx->status, 0, sizeof(uint32_t), 0)) != cudaSuccess)
@@ -906,6 +933,7 @@ static DenseParams dense_params(tpa_ctx* ctx, const Slot* sl, const PlanLayout& 
   DenseParams dp{};
   dp.tmap_k = ctx->tmap_k;
   dp.tmap_v = ctx->tmap_v;
+  dp.run_maps = ctx->run_maps;
   dp.q = static_cast<const __nv_bfloat16*>(q);
   dp.out = static_cast<__nv_bfloat16*>(out);
   dp.lse = lse;

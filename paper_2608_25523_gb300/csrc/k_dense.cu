@@ -20,18 +20,21 @@
 // A CTA owns one SM (198 KB of shared memory).  The first n_dense_ctas CTAs
 // walk their share of the dense items (longest first, snake order), holding
 // 512 TMEM columns; the rest run split-KV warps on the same shared memory.
-//   warp 0      TMA producer: K and V tiles (8 pages, one 128B-swizzled box
-//               per page and operand) into a 2-stage ring, running ahead
-//               across item boundaries; lane i loads page i's id three tiles
-//               ahead and issues that page's boxes
+//   warps 0, 10 TMA producers of K and V: tiles of 8 pages into a 2-stage
+//               ring each, running ahead across item boundaries; lane i
+//               loads page i's id three tiles ahead.  A full tile on 8
+//               consecutive pages is one 128B-swizzled box of the kv head's
+//               page-run view, otherwise each lane issues its page's box
 //   warp 1      TMEM owner; one lane issues tcgen05.mma, whichever of QK /
 //               PV is ready first (QK may run two tiles ahead of PV):
 //                 S_j = Q K_j^T  (M=128, N=128 keys, K=d)   into TMEM S[j%2]
-//                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O
+//                 O  += P_j V_j  (M=128, N=d, K=128 keys)   into TMEM O, with P_j
+//                                read from TMEM P[j%2] and V_j from shared memory
 //   warps 2..9  warp w owns TMEM lane quarter w % 4 (rows 32(w%4)..+31) and
 //               key half (w-2)/4.  Per tile: read S, take the full-row max
 //               (both warps of a pair, so their running max agrees without
-//               synchronising), write P for their key half, rescale O in
+//               synchronising), write P (bf16) for their key half into
+//               TMEM, rescale O in
 //               TMEM only when the max grew by more than 2^8 (otherwise the
 //               stale max stays the reference, which is exact: it is only a
 //               stabiliser); then the item's epilogue.  The next item's Q
@@ -50,7 +53,8 @@ namespace {
 
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
-constexpr int kThreads = 320;               // producer, MMA, 8 softmax warps
+constexpr int kThreads = 352;               // K producer, MMA, 8 softmax warps, V producer
+constexpr int kWarpV = 10;                  // the V producer warp
 constexpr int kSoftmax = 256;
 
 __device__ __forceinline__ float fast_exp2(float x) {
@@ -61,27 +65,32 @@ __device__ __forceinline__ float fast_exp2(float x) {
 
 __device__ __forceinline__ void softmax_bar() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
 
+constexpr int kSplitWarps = 8;
+constexpr int kSplitStages = 3;
+
 template <int D>
 struct DenseCfg {
   static constexpr int NCH = D / 64;               // 64-dim chunks of a 128-byte row
   static constexpr int kChunk = 128 * 128;         // one chunk of a 128-row/128-key tile
   static constexpr int kQBytes = NCH * kChunk;     // Q   [chunk][row][128 B]
-  static constexpr int kPBytes = 2 * kChunk;       // P   [key chunk][row][128 B]
   static constexpr int kKVBytes = NCH * kChunk;    // K,V 8 pages, see kv_off
   static constexpr int kPageBytes = NCH * 2048;    // one page of one kv head
   static constexpr int kGroup = NCH * 1024;        // stride of 8-key groups
   static constexpr int kStages = 2;
   static constexpr int kOffQ = 0;
-  static constexpr int kOffP = kOffQ + kQBytes;
-  static constexpr int kOffK = kOffP + 2 * kPBytes;  // P is double-buffered
+  static constexpr int kOffK = kOffQ + kQBytes;
   static constexpr int kOffV = kOffK + kStages * kKVBytes;
   static constexpr int kOffBar = kOffV + kStages * kKVBytes;
   static constexpr int kNumBars = 18;
   static constexpr int kOffL = kOffBar + kNumBars * 8;   // partial row sums [2][128]
   static constexpr int kOffMisc = kOffL + 2 * 128 * 4;
-  static constexpr int kSmem = 1024 + kOffMisc + 64;
+  // split-KV CTAs of the same launch lay out their page rings from the start
+  static constexpr int kSplitSmem =
+      kSplitWarps * (SplitCfg<D, kSplitStages>::kWarpBytes + kSplitStages * 8) + 16;
+  static constexpr int kSmem = 1024 + (kOffMisc + 64 > kSplitSmem ? kOffMisc + 64 : kSplitSmem);
   static constexpr uint32_t kTmemCols = 512;
-  static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
+  // TMEM: S double buffer, O, then P double buffer (bf16, two per column)
+  static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256, kColP = 256 + D;
 };
 
 // barrier slots
@@ -116,14 +125,12 @@ __device__ __forceinline__ int item_of(int k, int g) {
 
 // Split-KV role of a CTA of the same launch: 8 independent warps, each with
 // a 3-stage TMA page ring in the shared memory the dense role would use.
-constexpr int kSplitWarps = 8;
-constexpr int kSplitStages = 3;
 
 template <int D, int G>
 __device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) {
   using W = SplitCfg<D, kSplitStages>;
-  static_assert(kSplitWarps * (W::kWarpBytes + kSplitStages * 8) + 16 <= DenseCfg<D>::kOffMisc,
-                "split-KV rings fit in the dense role's shared memory");
+  static_assert(kSplitWarps * (W::kWarpBytes + kSplitStages * 8) + 16 <= DenseCfg<D>::kSmem - 1024,
+                "split-KV rings fit in the launch's shared memory");
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= kSplitWarps) return;
@@ -198,18 +205,27 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     prefetch_tmap(&p.tmap_k);
     prefetch_tmap(&p.tmap_v);
   }
+  if (threadIdx.x >= 32 && threadIdx.x < 32 + 2 * p.hkv && p.run_maps)
+    prefetch_tmap(p.run_maps + (threadIdx.x - 32));
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer
-    // Lane i (< 8) owns page i of every tile: it loads that page id ahead and
-    // issues the page's TMA boxes, so a tile's boxes go out from 8 lanes at
-    // once.  Lane 0 posts the expected byte count first.
-    int kph_last[2] = {-1, -1}, vph_last[2] = {-1, -1};
+  if (warp == 0 || warp == kWarpV) {
+    // ------------------------------------------------------------ producers
+    // Warp 0 streams K, warp kWarpV streams V, each through its own 2-stage
+    // ring, so K runs ahead of the PV pipeline.  Lane i (< 8) owns page i of
+    // every tile: it loads that page id ahead and issues the page's TMA box,
+    // so a tile's boxes go out from 8 lanes at once.  Lane 0 posts the
+    // expected byte count first.
+    const bool is_v = warp == kWarpV;
+    uint64_t* const full = bars + (is_v ? B_VFULL : B_KFULL);
+    uint64_t* const empty = bars + (is_v ? B_VEMPTY : B_KEMPTY);
+    const CUtensorMap* const tmap = is_v ? &p.tmap_v : &p.tmap_k;
+    uint8_t* const ring = smem + (is_v ? C::kOffV : C::kOffK);
+    int ph_last[2] = {-1, -1};
     bool pok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
       return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
@@ -254,22 +270,24 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         pid1 = pid2;
         pid2 = page_id(item, j + 3);
         const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
-        if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(p.status, kStatusBadPage);
+        if (__any_sync(0xffffffffu, bad) && lane == 0 && !is_v) atomicOr(p.status, kStatusBadPage);
         const int z = (bad ? 0 : pid) * p.hkv + item.kv_head;
-        if (!wait_all(&bars[B_KEMPTY + s], ph ^ 1u)) { pok = false; break; }
-        if (lane == 0) mbar_arrive_expect_tx(&bars[B_KFULL + s], bytes);
+        // a full tile on 8 consecutive pages goes as one box of the kv head's
+        // page-run view; otherwise one box per page
+        const int32_t pid_0 = __shfl_sync(0xffffffffu, pid, 0);
+        const bool run = npg == 8 &&
+                         __all_sync(0xffffffffu, lane >= 8 || (!bad && pid == pid_0 + lane));
+        if (!wait_all(&empty[s], ph ^ 1u)) { pok = false; break; }
+        if (lane == 0) mbar_arrive_expect_tx(&full[s], bytes);
         __syncwarp();
-        if (lane < npg)
-          tma_load_5d(smem + C::kOffK + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_k,
-                      &bars[B_KFULL + s], 0, 0, 0, 0, z);
-        kph_last[s] = static_cast<int>(ph);
-        if (!wait_all(&bars[B_VEMPTY + s], ph ^ 1u)) { pok = false; break; }
-        if (lane == 0) mbar_arrive_expect_tx(&bars[B_VFULL + s], bytes);
-        __syncwarp();
-        if (lane < npg)
-          tma_load_5d(smem + C::kOffV + s * C::kKVBytes + lane * C::kPageBytes, &p.tmap_v,
-                      &bars[B_VFULL + s], 0, 0, 0, 0, z);
-        vph_last[s] = static_cast<int>(ph);
+        if (run) {
+          if (lane == 0)
+            tma_load_5d(ring + s * C::kKVBytes, p.run_maps + (is_v ? p.hkv : 0) + item.kv_head,
+                        &full[s], 0, 0, 0, 0, pid_0);
+        } else if (lane < npg) {
+          tma_load_5d(ring + s * C::kKVBytes + lane * C::kPageBytes, tmap, &full[s], 0, 0, 0, 0, z);
+        }
+        ph_last[s] = static_cast<int>(ph);
         if (has_next && j == 0) nitem = p.items[idx_n];
         if (has_next && j == 1) {
           n0 = page_id(nitem, 0);
@@ -297,10 +315,8 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     if (*abort_flag && lane == 0) {
       // let every issued copy land before the CTA's shared memory goes away
       volatile int never = 0;
-      for (int s = 0; s < 2; ++s) {
-        if (kph_last[s] >= 0) (void)mbar_wait(&bars[B_KFULL + s], kph_last[s], &never);
-        if (vph_last[s] >= 0) (void)mbar_wait(&bars[B_VFULL + s], vph_last[s], &never);
-      }
+      for (int s = 0; s < 2; ++s)
+        if (ph_last[s] >= 0) (void)mbar_wait(&full[s], ph_last[s], &never);
     }
     __syncwarp();  // the warp reaches the teardown barrier converged
   } else if (warp == 1) {
@@ -309,7 +325,6 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       constexpr uint32_t idesc_qk = umma_idesc_bf16(128, 128, false, false);
       constexpr uint32_t idesc_pv = umma_idesc_bf16(128, D, false, true);
       const uint32_t qbase = smem_u32(smem + C::kOffQ);
-      const uint32_t pbase = smem_u32(smem + C::kOffP);
       const uint32_t kbase0 = smem_u32(smem + C::kOffK);
       const uint32_t vbase0 = smem_u32(smem + C::kOffV);
       auto issue_qk = [&](int g) {
@@ -330,12 +345,11 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         const int s = g & 1;
         tc_fence_after();
         const uint32_t vb = vbase0 + s * C::kKVBytes;
+        const uint32_t pcol = tmem + C::kColP + (g & 1) * 64;  // P from TMEM, 8 columns per 16 keys
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t a = umma_sdesc(pbase + (g & 1) * C::kPBytes + (kk >> 2) * C::kChunk +
-                                            (kk & 3) * 32, 16, 1024);
           const uint64_t b = umma_sdesc(vb + kk * C::kPageBytes, 1024, C::kGroup);
-          umma_bf16_ss(tmem + C::kColO, a, b, idesc_pv, (!first || kk > 0) ? 1u : 0u);
+          umma_bf16_ts(tmem + C::kColO, pcol + kk * 8, b, idesc_pv, (!first || kk > 0) ? 1u : 0u);
         }
         umma_commit(&bars[B_PVDONE + (g & 1)]);
         umma_commit(&bars[B_VEMPTY + s]);
@@ -410,7 +424,6 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     const int own = half * 64;   // first S column of this thread's key half
     const int other = 64 - own;
     const float sc = p.scale_log2;
-    uint8_t* ps = smem + C::kOffP;
     bool ok = true;
     // warp-uniform outcome, so .sync.aligned tcgen05 ops never see a split warp
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
@@ -587,17 +600,16 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
             }
           }
         }
-        // this half of the P row: keys own .. own+63 = P chunk `half`
+        // this half of the P row (keys own .. own+63) into TMEM P buffer g % 2:
+        // 32 columns of two bf16 each, in key order
+        {
+          float pk[32];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          uint4 v;
-          v.x = pack_bf16(x[8 * u + 0], x[8 * u + 1]);
-          v.y = pack_bf16(x[8 * u + 2], x[8 * u + 3]);
-          v.z = pack_bf16(x[8 * u + 4], x[8 * u + 5]);
-          v.w = pack_bf16(x[8 * u + 6], x[8 * u + 7]);
-          *reinterpret_cast<uint4*>(ps + (g & 1) * C::kPBytes + half * C::kChunk + swz128(row, u)) = v;
+          for (int u = 0; u < 32; ++u) pk[u] = __uint_as_float(pack_bf16(x[2 * u], x[2 * u + 1]));
+          tmem_st32(tmem + lane_base + C::kColP + (g & 1) * 64 + half * 32, pk);
+          tmem_wait_st();
         }
-        fence_proxy_async();
+        if (t.nvalid < 128) fence_proxy_async();  // the zeroed V rows, before the PV reads them
         tc_fence_before();
         mbar_arrive(&bars[B_PFULL + (g & 1)]);
       }

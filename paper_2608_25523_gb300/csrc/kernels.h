@@ -33,6 +33,10 @@ cudaError_t launch_page_copy(const int32_t* pages, int len, int to_pages, const 
 struct DenseParams {
   CUtensorMap tmap_k;  // 5-D view of the K pool: one box = one page of one kv head
   CUtensorMap tmap_v;
+  // Device array of 2 * hkv 5-D views, K then V, one per kv head, whose
+  // last dimension steps over whole pages: one box = 8 consecutive pages of
+  // that kv head (a full tile whose pages are contiguous in the pool).
+  const CUtensorMap* run_maps;
   const __nv_bfloat16* q;
   __nv_bfloat16* out;
   float* lse;
