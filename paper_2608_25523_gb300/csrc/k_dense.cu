@@ -20,7 +20,7 @@
 // A CTA owns one SM (198 KB of shared memory).  The first n_dense_ctas CTAs
 // walk their share of the dense items (longest first, snake order), holding
 // 512 TMEM columns; the rest run split-KV warps on the same shared memory.
-//   warps 0, 10 TMA producers of K and V: tiles of 8 pages into a 2-stage
+//   warps 0, 10 TMA producers of K and V: tiles of 8 pages into a 3-stage
 //               ring each, running ahead across item boundaries; lane i
 //               loads page i's id three tiles ahead.  A full tile on 8
 //               consecutive pages is one 128B-swizzled box of the kv head's
@@ -76,12 +76,12 @@ struct DenseCfg {
   static constexpr int kKVBytes = NCH * kChunk;    // K,V 8 pages, see kv_off
   static constexpr int kPageBytes = NCH * 2048;    // one page of one kv head
   static constexpr int kGroup = NCH * 1024;        // stride of 8-key groups
-  static constexpr int kStages = 2;
+  static constexpr int kStages = 3;   // K and V ring depth
   static constexpr int kOffQ = 0;
   static constexpr int kOffK = kOffQ + kQBytes;
   static constexpr int kOffV = kOffK + kStages * kKVBytes;
   static constexpr int kOffBar = kOffV + kStages * kKVBytes;
-  static constexpr int kNumBars = 18;
+  static constexpr int kNumBars = 22;
   static constexpr int kOffL = kOffBar + kNumBars * 8;   // partial row sums [2][128]
   static constexpr int kOffMisc = kOffL + 2 * 128 * 4;
   // split-KV CTAs of the same launch lay out their page rings from the start
@@ -94,8 +94,8 @@ struct DenseCfg {
 };
 
 // barrier slots
-enum { B_KFULL = 0, B_KEMPTY = 2, B_VFULL = 4, B_VEMPTY = 6, B_SFULL = 8, B_SFREE = 10,
-       B_PFULL = 12, B_PVDONE = 14, B_QFULL = 16, B_DRAIN = 17 };
+enum { B_KFULL = 0, B_KEMPTY = 3, B_VFULL = 6, B_VEMPTY = 9, B_SFULL = 12, B_SFREE = 14,
+       B_PFULL = 16, B_PVDONE = 18, B_QFULL = 20, B_DRAIN = 21 };
 
 struct TileInfo {
   int key0;     // first key of the tile within its segment
@@ -187,11 +187,13 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   // ---------------------------------------------------------------- setup
   if (threadIdx.x == 0) {
     *abort_flag = 0;
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < C::kStages; ++i) {
       mbar_init(&bars[B_KFULL + i], 1);
       mbar_init(&bars[B_KEMPTY + i], 1);
       mbar_init(&bars[B_VFULL + i], 1);
       mbar_init(&bars[B_VEMPTY + i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(&bars[B_SFULL + i], 1);
       mbar_init(&bars[B_SFREE + i], kSoftmax);
     }
@@ -215,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
 
   if (warp == 0 || warp == kWarpV) {
     // ------------------------------------------------------------ producers
-    // Warp 0 streams K, warp kWarpV streams V, each through its own 2-stage
+    // Warp 0 streams K, warp kWarpV streams V, each through its own 3-stage
     // ring, so K runs ahead of the PV pipeline.  Lane i (< 8) owns page i of
     // every tile: it loads that page id ahead and issues the page's TMA box,
     // so a tile's boxes go out from 8 lanes at once.  Lane 0 posts the
@@ -225,7 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     uint64_t* const empty = bars + (is_v ? B_VEMPTY : B_KEMPTY);
     const CUtensorMap* const tmap = is_v ? &p.tmap_v : &p.tmap_k;
     uint8_t* const ring = smem + (is_v ? C::kOffV : C::kOffK);
-    int ph_last[2] = {-1, -1};
+    int ph_last[C::kStages] = {-1, -1, -1};
     bool pok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
       return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
@@ -261,8 +263,8 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       int32_t pid0 = f0, pid1 = f1, pid2 = f2;
       for (int j = 0; j < ntiles; ++j, ++gt) {
         const TileInfo t = tile_at(item, j);
-        const int s = gt & 1;
-        const uint32_t ph = (gt >> 1) & 1;
+        const int s = gt % C::kStages;
+        const uint32_t ph = (gt / C::kStages) & 1;
         const int npg = (t.nvalid + kPage - 1) / kPage;
         const uint32_t bytes = static_cast<uint32_t>(npg * C::kPageBytes);
         const int32_t pid = pid0;
@@ -315,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     if (*abort_flag && lane == 0) {
       // let every issued copy land before the CTA's shared memory goes away
       volatile int never = 0;
-      for (int s = 0; s < 2; ++s)
+      for (int s = 0; s < C::kStages; ++s)
         if (ph_last[s] >= 0) (void)mbar_wait(&full[s], ph_last[s], &never);
     }
     __syncwarp();  // the warp reaches the teardown barrier converged
@@ -328,9 +330,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       const uint32_t kbase0 = smem_u32(smem + C::kOffK);
       const uint32_t vbase0 = smem_u32(smem + C::kOffV);
       auto issue_qk = [&](int g) {
-        const int s = g & 1;
+        const int s = g & 1;            // S buffer
+        const int ks = g % C::kStages;  // K stage
         tc_fence_after();
-        const uint32_t kb = kbase0 + s * C::kKVBytes;
+        const uint32_t kb = kbase0 + ks * C::kKVBytes;
         const uint32_t scol = s ? C::kColS1 : C::kColS0;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
@@ -339,12 +342,12 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           umma_bf16_ss(tmem + scol, a, b, idesc_qk, kk > 0 ? 1u : 0u);
         }
         umma_commit(&bars[B_SFULL + s]);
-        umma_commit(&bars[B_KEMPTY + s]);
+        umma_commit(&bars[B_KEMPTY + ks]);
       };
       auto issue_pv = [&](int g, bool first) {
-        const int s = g & 1;
+        const int ks = g % C::kStages;  // V stage
         tc_fence_after();
-        const uint32_t vb = vbase0 + s * C::kKVBytes;
+        const uint32_t vb = vbase0 + ks * C::kKVBytes;
         const uint32_t pcol = tmem + C::kColP + (g & 1) * 64;  // P from TMEM, 8 columns per 16 keys
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
@@ -352,7 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           umma_bf16_ts(tmem + C::kColO, pcol + kk * 8, b, idesc_pv, (!first || kk > 0) ? 1u : 0u);
         }
         umma_commit(&bars[B_PVDONE + (g & 1)]);
-        umma_commit(&bars[B_VEMPTY + s]);
+        umma_commit(&bars[B_VEMPTY + ks]);
       };
       bool ok = true;
       int gt = 0;
@@ -373,9 +376,8 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           bool progressed = false;
           if (nq < ntiles && nq <= np + 2) {
             const int g = gt + nq;
-            const int s = g & 1;
-            const uint32_t ph = (g >> 1) & 1;
-            if (mbar_test(&bars[B_KFULL + s], ph) && mbar_test(&bars[B_SFREE + s], ph ^ 1u)) {
+            if (mbar_test(&bars[B_KFULL + g % C::kStages], (g / C::kStages) & 1) &&
+                mbar_test(&bars[B_SFREE + (g & 1)], ((g >> 1) & 1) ^ 1u)) {
               issue_qk(g);
               ++nq;
               progressed = true;
@@ -384,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           if (np < nq) {
             const int g = gt + np;
             if (mbar_test(&bars[B_PFULL + (g & 1)], (g >> 1) & 1) &&
-                mbar_test(&bars[B_VFULL + (g & 1)], (g >> 1) & 1)) {
+                mbar_test(&bars[B_VFULL + g % C::kStages], (g / C::kStages) & 1)) {
               issue_pv(g, np == 0);
               ++np;
               progressed = true;
@@ -584,9 +586,9 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         if (t.nvalid < 128) {
           // keys past the range: zero their V rows (stale data may not be finite);
           // each half zeroes its own 64-dim chunk (or its half of the only chunk)
-          if (!wait_all(&bars[B_VFULL + s], (g >> 1) & 1)) { ok = false; break; }
+          if (!wait_all(&bars[B_VFULL + g % C::kStages], (g / C::kStages) & 1)) { ok = false; break; }
           if (row >= t.nvalid) {
-            uint8_t* vst = smem + C::kOffV + s * C::kKVBytes;
+            uint8_t* vst = smem + C::kOffV + (g % C::kStages) * C::kKVBytes;
             if (C::NCH == 2) {
 #pragma unroll
               for (int u = 0; u < 8; ++u)
