@@ -1016,10 +1016,12 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     // ranges; level 2 (split-KV CTAs): the suffixes.  The split count and the
     // number of dense CTAs are chosen together so that every dense CTA gets
     // the same whole number m of (near-equal) items while the split-KV CTAs
-    // finish at about the same time.  Rates measured on GB300 with both
-    // roles streaming: a dense 128x128 tile ~2 us, plus ~2 us per item (the
-    // next item's Q is loaded once the previous item's last QK is done);
-    // split-KV ~50 GB/s of KV per SM.  Ties go to fewer splits.
+    // finish at about the same time: the dense level is tensor-heavy and the
+    // split level HBM-heavy, so the two run side by side (a dense CTA that is
+    // done early still joins the split-KV work).  Rates measured on GB300
+    // with both roles streaming: a dense 128x128 tile ~2 us, plus ~2 us per
+    // item (the next item's Q is loaded once the previous item's last QK is
+    // done); split-KV ~50 GB/s of KV per SM.  Ties go to fewer splits.
     constexpr double kTileUs = 2.0, kItemUs = 2.0, kSplitBytesPerUs = 50e3;
     double split_bytes = 0;
     for (int i = 0; i < n; ++i) split_bytes += static_cast<double>(keys_of(i)) * hkv * 4.0 * ctx->d;

@@ -17,9 +17,10 @@
 //    request's chunk attends to the whole prefix and causally to the
 //    request's own suffix, writing final outputs directly.
 //
-// A CTA owns one SM (198 KB of shared memory).  The first n_dense_ctas CTAs
+// A CTA owns one SM (226 KB of shared memory).  The first n_dense_ctas CTAs
 // walk their share of the dense items (longest first, snake order), holding
-// 512 TMEM columns; the rest run split-KV warps on the same shared memory.
+// 512 TMEM columns, and then join the split-KV work; the rest run split-KV
+// warps from the start on the same shared memory.
 //   warps 0, 10 TMA producers of K and V: tiles of 8 pages into a 3-stage
 //               ring each, running ahead across item boundaries; lane i
 //               loads page i's id three tiles ahead.  A full tile on 8
@@ -683,6 +684,12 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, C::kTmemCols);
+  }
+  // Decode: this CTA's dense items are done (every copy it issued has been
+  // consumed), so its warps join the split-KV work on the same shared memory.
+  if (p.n_sitems > 0) {
+    __syncthreads();
+    if (!*abort_flag) split_role<D, G>(p, smem);
   }
 }
 

@@ -7,9 +7,7 @@
 // Hq/Hkv query rows of one token against one key range of one page run (a
 // request suffix, or in the flat cross-check mode also a prefix); it yields
 // a partial (o, lse).  In the cascade decode the item holding a request's
-// last key first appends the step's token to the pool, and the item that
-// completes the last partial of a (token, kv head) merges all of them by
-// log-sum-exp.
+// last key first appends the step's token to the pool.
 //
 // Design (memory-bound: ~4 flop per KV byte at G=4):
 //  * each page of one kv head is one TMA box per operand (128-byte swizzle)
@@ -19,7 +17,10 @@
 //    accumulators as the A operand (no shared-memory round trip); V comes
 //    through ldmatrix.trans;
 //  * online softmax in base 2 with fp32 accumulators;
-//  * warps pull items from an atomic counter (items sorted longest first).
+//  * warps pull items from an atomic counter (items sorted longest first);
+//    a warp claims and resolves its next item, appends its token and loads
+//    its page ids while the current one streams, and keeps its ring full
+//    across the item boundary, so items cost no extra load latency.
 #pragma once
 #include "kernels.h"
 #include "ptx.cuh"
@@ -72,20 +73,22 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
-// Work item `idx` (explicit, or derived from the per-token records).
+// Work item `idx` (explicit, or derived from the per-token records).  Called
+// by the whole warp.
 __device__ __forceinline__ SuffixItem fetch_item(const SplitArgs& a, int idx) {
   if (a.items) return a.items[idx];
   const int u = idx / a.hkv;
   int tok, s, k0, k1;
   if (u < a.n_full) {
-    int lo = 0, hi = a.n_tok;  // full_prefix[lo] <= u < full_prefix[hi]
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      if (__ldg(a.full_prefix + mid) <= u) lo = mid;
-      else hi = mid;
+    // the token is the number of i in [1, n_tok) with full_prefix[i] <= u
+    // (full_prefix is non-decreasing): the lanes test 32 entries a round
+    const int lane = threadIdx.x & 31;
+    tok = 0;
+    for (int i0 = 1; i0 < a.n_tok; i0 += 32) {
+      const int i = i0 + lane;
+      tok += __popc(__ballot_sync(0xffffffffu, i < a.n_tok && __ldg(a.full_prefix + i) <= u));
     }
-    tok = lo;
-    s = u - __ldg(a.full_prefix + lo);
+    s = u - __ldg(a.full_prefix + tok);
     k0 = s * a.split_keys;
     k1 = k0 + a.split_keys;
   } else {
@@ -122,24 +125,28 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
   const int gq = lane >> 2;  // mma group: query row of this lane
   const int tig = lane & 3;  // thread in group
   uint32_t it = 0;           // pages consumed by this warp so far (ring position)
-  uint32_t issued = 0;       // pages issued by this warp so far
+  uint32_t issued = 0;       // pages issued by this warp so far (lane 0's count, broadcast)
   bool failed = false;
 
-  while (!failed) {
-    int idx = 0;
-    if (lane == 0) idx = static_cast<int>(atomicAdd(a.queue, 1u));
-    idx = __shfl_sync(0xffffffffu, idx, 0);
-    if (idx >= a.n_items) break;
-    const SuffixItem item = fetch_item(a, idx);
-    const int npg = (item.n_keys + kPage - 1) / kPage;
-
-    if (item.app_src >= 0 && a.k_new) {
-      // append the step's token to the pool before its page is loaded
+  // An item with its page ids: lane i holds pages i and i + 32 of its run.
+  struct Work {
+    SuffixItem item;
+    int npg;
+    int32_t pid0, pid1;
+  };
+  auto load_work = [&](int idx, Work& w) {  // whole warp
+    w.item = fetch_item(a, idx);
+    w.npg = (w.item.n_keys + kPage - 1) / kPage;
+    w.pid0 = lane < w.npg ? __ldg(a.pages + w.item.pages + lane) : 0;
+    w.pid1 = lane + 32 < w.npg ? __ldg(a.pages + w.item.pages + lane + 32) : 0;
+    if (w.item.app_src >= 0 && a.k_new) {
+      // append the step's token to the pool before its page is loaded (its
+      // page belongs to this item alone: key ranges start on page boundaries)
       constexpr int U = D / 8;  // 16-byte units of one row
-      const int64_t pg = item.app_dst / kPage;
+      const int64_t pg = w.item.app_dst / kPage;
       if (pg >= 0 && pg < a.num_pages) {
-        const int64_t src = (static_cast<int64_t>(item.app_src) * a.hkv + item.kv_head) * D;
-        const int64_t dst = ((pg * a.hkv + item.kv_head) * kPage + item.app_dst % kPage) * D;
+        const int64_t src = (static_cast<int64_t>(w.item.app_src) * a.hkv + w.item.kv_head) * D;
+        const int64_t dst = ((pg * a.hkv + w.item.kv_head) * kPage + w.item.app_dst % kPage) * D;
         for (int u = lane; u < 2 * U; u += 32) {
           const bool isv = u >= U;
           const int uu = isv ? u - U : u;
@@ -152,6 +159,44 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
       asm volatile("fence.proxy.async.global;" ::: "memory");
       __syncwarp();
     }
+  };
+  // TMA page `pg` of `w` into ring slot issued % S (whole warp; lane 0 issues)
+  auto issue = [&](const Work& w, int pg) {
+    int64_t pid = pg < 32   ? __shfl_sync(0xffffffffu, w.pid0, pg)
+                  : pg < 64 ? __shfl_sync(0xffffffffu, w.pid1, pg - 32)
+                            : static_cast<int64_t>(__ldg(a.pages + w.item.pages + pg));
+    if (lane == 0) {
+      const int st = static_cast<int>(issued % S);
+      uint8_t* kst = ring + st * C::kStageBytes;
+      uint8_t* vst = kst + C::kPageBytes;
+      if (pid < 0 || pid >= a.num_pages) {
+        atomicOr(a.status, kStatusBadPage);
+        pid = 0;
+      }
+      const int z = static_cast<int>(pid * a.hkv + w.item.kv_head);
+      fence_proxy_async();
+      mbar_arrive_expect_tx(&bars[st], 2 * C::kPageBytes);
+      tma_load_5d(kst, a.tmap_k, &bars[st], 0, 0, 0, 0, z);
+      tma_load_5d(vst, a.tmap_v, &bars[st], 0, 0, 0, 0, z);
+    }
+    ++issued;
+  };
+  auto claim = [&]() -> uint32_t { return lane == 0 ? atomicAdd(a.queue, 1u) : 0u; };
+
+  int idx = __shfl_sync(0xffffffffu, static_cast<int>(claim()), 0);
+  Work cur{};
+  int cur_iss = 0;  // pages of cur issued
+  if (idx < a.n_items) {
+    load_work(idx, cur);
+    while (cur_iss < cur.npg && cur_iss < S) issue(cur, cur_iss++);
+  }
+
+  while (idx < a.n_items) {
+    const uint32_t ticket = claim();  // the next item, claimed while this one streams
+    Work nxt{};
+    int nxt_iss = 0;
+    int idx_n = a.n_items;
+    const SuffixItem& item = cur.item;
 
     // Query fragments (A operand): rows >= G and the upper 8 rows are zero.
     uint32_t qa[D / 16][2];
@@ -166,35 +211,12 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
       }
     }
 
-    auto issue = [&](int pg) {  // lane 0: TMA page `pg` of the item into ring slot issued % S
-      const int st = static_cast<int>(issued % S);
-      uint8_t* kst = ring + st * C::kStageBytes;
-      uint8_t* vst = kst + C::kPageBytes;
-      int64_t pid = a.pages[item.pages + pg];
-      if (pid < 0 || pid >= a.num_pages) {
-        atomicOr(a.status, kStatusBadPage);
-        pid = 0;
-      }
-      const int z = static_cast<int>(pid * a.hkv + item.kv_head);
-      fence_proxy_async();
-      mbar_arrive_expect_tx(&bars[st], 2 * C::kPageBytes);
-      tma_load_5d(kst, a.tmap_k, &bars[st], 0, 0, 0, 0, z);
-      tma_load_5d(vst, a.tmap_v, &bars[st], 0, 0, 0, 0, z);
-      ++issued;
-    };
-
-    if (lane == 0) {
-      const int pre = npg < S ? npg : S;
-      for (int i = 0; i < pre; ++i) issue(i);
-    }
-    issued = __shfl_sync(0xffffffffu, issued, 0);
-
     float o[D / 8][4];
 #pragma unroll
     for (int nt = 0; nt < D / 8; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
     float m = -INFINITY, l = 0.f;
 
-    for (int pg = 0; pg < npg; ++pg) {
+    for (int pg = 0; pg < cur.npg; ++pg) {
       const uint32_t cnt = it + pg;
       const int st = static_cast<int>(cnt % S);
       if (!__all_sync(0xffffffffu, mbar_wait(&bars[st], (cnt / S) & 1u, abort_flag))) {
@@ -270,11 +292,17 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
         }
       }
       __syncwarp();
-      if (lane == 0 && pg + S < npg) issue(pg + S);
-      issued = __shfl_sync(0xffffffffu, issued, 0);
+      if (pg == 0) {
+        // resolve the next item now: its loads overlap this item's stream
+        idx_n = __shfl_sync(0xffffffffu, static_cast<int>(ticket), 0);
+        if (idx_n < a.n_items) load_work(idx_n, nxt);
+      }
+      // refill the slot this page freed: this item's next page, else the next item's
+      if (cur_iss < cur.npg) issue(cur, cur_iss++);
+      else if (nxt_iss < nxt.npg) issue(nxt, nxt_iss++);
     }
     if (failed) break;
-    it += npg;
+    it += cur.npg;
 
     l += __shfl_xor_sync(0xffffffffu, l, 1);
     l += __shfl_xor_sync(0xffffffffu, l, 2);
@@ -289,6 +317,11 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
             make_float2(o[nt][0] * inv, o[nt][1] * inv);
       if (tig == 0) a.part_lse[slot] = (m + __log2f(l)) * kLn2;
     }
+
+    idx = idx_n;
+    cur = nxt;
+    cur_iss = nxt_iss;
+    while (issued - it < static_cast<uint32_t>(S) && cur_iss < cur.npg) issue(cur, cur_iss++);
   }
 
   if (failed) {
