@@ -149,6 +149,7 @@ __device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) 
     prefetch_tmap(&p.tmap_k);
     prefetch_tmap(&p.tmap_v);
   }
+  pdl_wait();  // no global memory was touched before this point
   SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, nullptr, p.n_sitems,
               p.stoks, p.full_prefix, p.tail_order, p.n_stok, p.n_full, p.split_keys, p.pages,
               p.squeue, p.status, p.num_pages, p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new,
@@ -176,7 +177,6 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       return;
     }
   }
-  pdl_wait();  // the kernel before this one (if a programmatic dependent) has completed
   if (static_cast<int>(blockIdx.x) >= p.n_dense_ctas) {
     split_role<D, G>(p, smem);
     return;
@@ -215,6 +215,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // The setup above touches only this CTA's shared and tensor memory; from
+  // here on the kernel before this one (if this is its programmatic
+  // dependent) must have completed.
+  pdl_wait();
 
   if (warp == 0 || warp == kWarpV) {
     // ------------------------------------------------------------ producers
