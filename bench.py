@@ -18,8 +18,10 @@ e2e    = the same metric through the public call with host buffers: the
          step's q / k_new / v_new come from pinned host memory and O / LSE
          go back, inside the timed region.
 Also reported (rank 0, N=1): the tcgen05 chunked-prefill workload
-(TFLOP/s), the mixed workload (reload + prefill + Zipf decode, ms/step)
-and the Llama-3-70B decode workload (GB/s), each with its own roofline.
+(TFLOP/s), the mixed workload (reload + prefill + Zipf decode, ms/step),
+the Llama-3-70B decode workload (GB/s), each with its own roofline, and the
+prefix-movement calibration (reload / offload bandwidth, the paper's
+mu / B_swap).
 
 Under torchrun every rank runs its own copy on its own GPU (the path has
 no exchange step: replicas only); value aggregates all ranks over the
@@ -112,6 +114,18 @@ def prefill_flops(w, chunks):
         # positions off..off+c-1 see lp prefix keys and p+1 suffix keys
         pairs += c * lp + c * off + c * (c + 1) // 2
     return pairs * w.num_q_heads * 4 * w.head_dim
+
+
+def job_rate(ms, units_per_rank, world, device):
+    """Slowest rank's timed region (max over ranks) and the whole-job rate:
+    the units all ranks processed over that time (per second)."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return ms, units_per_rank * world / (ms / 1e3)
 
 
 # ---------------------------------------------------------------- clocks --
@@ -225,13 +239,10 @@ def run_ours(args, rank, world, local_rank):
     ms = e0.elapsed_time(e1)
     barrier()
     clk = clocks.stop() if rank == 0 else None
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms, bytes_s = job_rate(ms, step_bytes * args.steps, world, dev)
     launches_per_step = s.ctx.query(B.Q_LAST_LAUNCHES)
     ms_step = ms / args.steps
-    value = step_bytes * args.steps * world / (ms / 1e3) / 1e9
+    value = bytes_s / 1e9
     tokens_s = n * args.steps * world / (ms / 1e3)
     status = s.ctx.device_status()
 
@@ -287,11 +298,8 @@ def run_ours(args, rank, world, local_rank):
     e1.record(stream)
     e1.synchronize()
     ms_e2e = e0.elapsed_time(e1)
-    if world > 1:
-        tt = torch.tensor([ms_e2e], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_e2e = float(tt.item())
-    e2e = {"value": round(step_bytes * e2e_steps * world / (ms_e2e / 1e3) / 1e9, 1), "unit": "GB/s",
+    ms_e2e, e2e_bytes_s = job_rate(ms_e2e, step_bytes * e2e_steps, world, dev)
+    e2e = {"value": round(e2e_bytes_s / 1e9, 1), "unit": "GB/s",
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
            "ms_per_step": round(ms_e2e / e2e_steps, 4)}
 
@@ -327,6 +335,7 @@ def run_ours(args, rank, world, local_rank):
         result["prefill"] = bench_prefill(args, dev, tf_peak, peak_src)
         result["decode_70b"] = bench_70b(args, dev, hbm_peak, peak_src)
         result["mixed"] = bench_mixed(args, dev)
+        result["movement"] = bench_movement(args, dev)
     if rank == 0 and world == 1 and not args.no_cpu:
         result["cpu_baseline"] = cpu_baseline(budget_s=15.0)
     return result
@@ -487,6 +496,109 @@ def bench_mixed(args, dev):
             "device_status": st}
 
 
+def bench_movement(args, dev):
+    """Prefix movement between GPU and pinned host memory (Sec. IV, Eq. 7:
+    T_move = mu / B_swap x the moved prefix lengths; the same mu l_a / B_swap
+    prices reuse in Eq. 10).  For prefixes of the Llama-3-8B layer (mu = 4096
+    B per token) of several lengths: reload = host -> free, permuted pages on
+    a side stream; offload = pages -> host.  Each is fitted as t = t0 + bytes
+    / B and compared with a plain pinned copy of the same bytes."""
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+
+    hkv, d, hq = 8, 128, 32
+    mu = 2 * hkv * d * 2
+    sizes = [1024, 4096, 16384, 65536]
+    lmax = max(sizes)
+    ctx = B.allocate(num_q_heads=hq, num_kv_heads=hkv, head_dim=d, num_pages=lmax // 16 + 64,
+                     max_agents=len(sizes), max_requests=1, max_tokens=1024,
+                     max_seq_len=lmax + 64, page_order_seed=3, device=dev)
+    side = torch.cuda.Stream(device=dev)
+    g = torch.Generator().manual_seed(11)
+    hk = torch.randn(lmax, hkv, d, generator=g).to(torch.bfloat16).pin_memory()
+    hv = torch.randn(lmax, hkv, d, generator=g).to(torch.bfloat16).pin_memory()
+    ok = torch.empty_like(hk).pin_memory()
+    ov = torch.empty_like(hv).pin_memory()
+    dk = torch.empty(lmax, hkv, d, dtype=torch.bfloat16, device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn, before=None, reps=5):
+        ts = []
+        for _ in range(reps + 1):
+            if before:
+                before()
+            e0.record(side)
+            fn()
+            e1.record(side)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1) * 1e3)
+        return sorted(ts[1:])[len(ts[1:]) // 2]   # median, first run dropped
+
+    rows = []
+    for a, ell in enumerate(sizes):
+        ctx.prefix_register(a, ell)
+        ctx.prefix_write(a, hk[:ell], hv[:ell], side)
+        side.synchronize()
+
+        resident = [True]
+
+        def evict():       # untimed: free the pages (table only)
+            if resident[0]:
+                ctx.prefix_evict(a)
+                resident[0] = False
+
+        def reload():      # pinned host -> free (permuted) pages
+            ctx.prefix_reload(a, hk[:ell], hv[:ell], side)
+            resident[0] = True
+
+        def offload():     # pages -> pinned host, then evicted
+            ctx.prefix_offload(a, ok[:ell], ov[:ell], side)
+            resident[0] = False
+
+        def make_resident():
+            if not resident[0]:
+                reload()
+
+        def h2d():
+            dk[:ell].copy_(hk[:ell], non_blocking=True)
+            dk[:ell].copy_(hv[:ell], non_blocking=True)
+
+        def d2h():
+            ok[:ell].copy_(dk[:ell], non_blocking=True)
+            ov[:ell].copy_(dk[:ell], non_blocking=True)
+
+        with torch.cuda.stream(side):
+            t_re = timed(reload, before=evict)
+            t_off = timed(offload, before=make_resident)
+            side.synchronize()
+            exact = bool(torch.equal(ok[:ell].view(torch.int16), hk[:ell].view(torch.int16)) and
+                         torch.equal(ov[:ell].view(torch.int16), hv[:ell].view(torch.int16)))
+            t_h2d, t_d2h = timed(h2d), timed(d2h)
+        side.synchronize()
+        rows.append({"tokens": ell, "bytes": ell * mu, "reload_us": round(t_re, 1),
+                     "offload_us": round(t_off, 1), "h2d_copy_us": round(t_h2d, 1),
+                     "d2h_copy_us": round(t_d2h, 1), "round_trip_bit_exact": exact})
+        evict()
+
+    def fit(key):
+        xs = [r["bytes"] for r in rows]
+        ys = [r[key] for r in rows]
+        n = len(xs)
+        mx, my = sum(xs) / n, sum(ys) / n
+        slope = sum((x - mx) * (y - my) for x, y in zip(xs, ys)) / sum((x - mx) ** 2 for x in xs)
+        return {"B_gbs": round(1e-3 / slope, 1), "t0_us": round(my - slope * mx, 1)}
+
+    ctx.close()
+    res = {"workload": "prefix movement, llama3_8b layer (mu = 4096 B/token), prefixes of "
+                       + ", ".join(str(x) for x in sizes) + " tokens, permuted pool",
+           "rows": rows, "reload": fit("reload_us"), "offload": fit("offload_us"),
+           "h2d_copy": fit("h2d_copy_us"), "d2h_copy": fit("d2h_copy_us")}
+    res["mu_over_B_swap_ns_per_token"] = {
+        "reload": round(mu / (res["reload"]["B_gbs"] * 1e9) * 1e9, 3),
+        "offload": round(mu / (res["offload"]["B_gbs"] * 1e9) * 1e9, 3)}
+    return res
+
+
 # ------------------------------------------------------ oracle baseline --
 
 def _blas_threads():
@@ -588,7 +700,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed"],
+    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement"],
                     help="run just one of the extra workloads (1 GPU) and print its result")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -609,7 +721,8 @@ def main():
         hbm_peak, tf_peak, _, peak_src = peaks()
         fn = {"prefill": lambda: bench_prefill(args, dev, tf_peak, peak_src),
               "decode_70b": lambda: bench_70b(args, dev, hbm_peak, peak_src),
-              "mixed": lambda: bench_mixed(args, dev)}[args.only]
+              "mixed": lambda: bench_mixed(args, dev),
+              "movement": lambda: bench_movement(args, dev)}[args.only]
         print(json.dumps({"only": args.only, "result": fn()}))
         return
     if world > 1:
