@@ -241,15 +241,20 @@ enum {
 TPA_API int tpa_query(tpa_ctx* ctx, int32_t what, int32_t id, int64_t* value);
 
 enum {
-  TPA_OPT_DECODE_MODE = 0,      /* 0: cascade (default): one persistent tensor-core launch
-                                   over stacked prefix tiles and per-request suffixes, with the
-                                   KV append and the LSE merge inside; 1: flat cross-check --
-                                   KV append, every key (prefix included) through the split-KV
-                                   kernel, then a separate merge */
+  TPA_OPT_DECODE_MODE = 0,      /* 0: cascade (default): one persistent launch over stacked
+                                   prefix tiles (tensor cores) and per-request suffixes
+                                   (split-KV, with the KV append), then the LSE merge launched as
+                                   its programmatic dependent; 1: flat cross-check -- KV append,
+                                   every key (prefix included) through the split-KV kernel, then
+                                   the merge */
   TPA_OPT_PREFIX_SPLITS = 1,    /* cascade: key splits per stacked prefix tile; 0 = automatic */
-  TPA_OPT_SUFFIX_SPLIT_KEYS = 2,/* keys per suffix work item (cascade: rounded up to 128;
-                                   flat: multiple of 16); 0 = automatic */
-  TPA_OPT_KERNEL_TIMING = 4     /* 1: bracket every kernel with CUDA events (tpa_kernel_times) */
+  TPA_OPT_SUFFIX_SPLIT_KEYS = 2,/* keys per suffix work item, a multiple of 16; 0 = automatic */
+  TPA_OPT_KERNEL_TIMING = 4,    /* 1: bracket every kernel with CUDA events (tpa_kernel_times) */
+  TPA_OPT_TEST_PLAN_WAIT = 5    /* test hook, 1: the next cascade decode's kernel waits for a
+                                   plan flag that is never written, so every CTA gives up at the
+                                   device wait limit (2 s) without touching the pool and
+                                   tpa_device_status reports TIMEOUT.  The context stays usable;
+                                   truncate that call's requests back to their lengths before it */
 };
 TPA_API int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value);
 
@@ -267,7 +272,8 @@ TPA_API int tpa_kernel_times(tpa_ctx* ctx, int32_t n, double* total_ms, int64_t*
  * *status = 0 when no kernel reported a problem; otherwise a bit set:
  * 1 a dense-kernel wait timed out, 2 a suffix-kernel wait timed out,
  * 4 a page id outside the pool was met (the access was redirected to page
- * 0).  Returns TIMEOUT if bit 1 or 2 is set, CUDA on a CUDA error. */
+ * 0), 8 a kernel gave up waiting for its plan upload (it did no work).
+ * Returns TIMEOUT if bit 1, 2 or 8 is set, CUDA on a CUDA error. */
 TPA_API int tpa_device_status(tpa_ctx* ctx, void* stream, uint32_t* status);
 
 /* Thread-local message describing the last failed call on this thread. */

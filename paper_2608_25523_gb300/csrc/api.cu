@@ -157,6 +157,7 @@ struct tpa_ctx {
 
   // options and statistics
   int decode_mode = 0;
+  int test_plan_wait = 0;  // test hook: the next cascade decode waits for a flag never written
   int prefix_splits = 0;
   int suffix_split_keys = 0;
   int64_t last_dense = 0, last_suffix = 0, last_launches = 0;
@@ -1297,6 +1298,10 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
           KernelTimer kt(ctx, K_DENSE, s);
         dp.plan_flag = plan_flag;
         dp.plan_seq = ctx->seq;
+        if (ctx->test_plan_wait) {  // a value the flag word never takes
+          dp.plan_seq = ctx->seq | (1ull << 63);
+          ctx->test_plan_wait = 0;
+        }
         // a programmatic dependent of the previous step's merge on this stream
         CUDA_TRY(launch_dense(dp, n_split, ctx->d, G, true, s));
       }
@@ -1567,6 +1572,9 @@ int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
     case TPA_OPT_KERNEL_TIMING:
       ctx->timing = value ? 1 : 0;
       return TPA_OK;
+    case TPA_OPT_TEST_PLAN_WAIT:
+      ctx->test_plan_wait = value ? 1 : 0;
+      return TPA_OK;
     default: return fail(TPA_ERR_INVALID_ARG, "unknown option %d", option);
   }
 }
@@ -1596,7 +1604,7 @@ int tpa_device_status(tpa_ctx* ctx, void* stream, uint32_t* status) {
   CUDA_TRY(cudaStreamSynchronize(s));
   CUDA_TRY(cudaMemcpy(status, ctx->status, sizeof(uint32_t), cudaMemcpyDeviceToHost));
   CUDA_TRY(cudaMemset(ctx->status, 0, sizeof(uint32_t)));
-  if (*status & (kStatusDenseTimeout | kStatusSuffixTimeout))
+  if (*status & (kStatusDenseTimeout | kStatusSuffixTimeout | kStatusPlanTimeout))
     return fail(TPA_ERR_TIMEOUT, "a device-side wait timed out (status 0x%x)", *status);
   return TPA_OK;
 }

@@ -253,3 +253,28 @@ def test_reload_rejects_unpinned_host_memory():
         s.ctx.prefix_reload(0, hk, hk)
     assert e.value.code == B.TPA_ERR_INVALID_ARG
     assert s.ctx.query(B.Q_PREFIX_RESIDENT, 0) == 0
+
+
+def test_plan_wait_timeout_is_reported_and_context_recovers():
+    # A decode whose kernel never sees its plan (test hook: the flag it waits
+    # for is never written) gives up at the device wait limit; the host reads
+    # the timeout from the status word, and after truncating that step's
+    # requests back the next step is exact again.
+    w = small_case(77, hq=8, hkv=2, d=128, prefix_len=[300, 40], req_agent=[0, 0, 1, 0],
+                   req_ctx=[10, 200, 33, 0], req_prefill=[0] * 4, req_decode=[1] * 4)
+    t, s = _session(w)
+    ids, q, kn, vn = s.decode_inputs()
+    lens = [s.ctx.query(B.Q_SUFFIX_LEN, r) for r in ids]
+    out, lse = s.new_outputs(len(ids))
+    s.ctx.set_option(B.OPT_TEST_PLAN_WAIT, 1)
+    s.decode(ids, q, kn, vn, out, lse)
+    status = s.ctx.device_status()
+    assert status & 8, status
+    assert s.ctx.device_status() == 0          # the word was cleared
+    s.ctx.request_truncate(ids, lens)
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    ref = oracle.workload_decode(w, t)
+    o_ref, l_ref = stack_decode_ref(ref, range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "after a plan-wait timeout")
