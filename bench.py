@@ -19,9 +19,10 @@ e2e    = the same metric through the public call with host buffers: the
          go back, inside the timed region.
 Also reported (rank 0, N=1): the tcgen05 chunked-prefill workload
 (TFLOP/s), the mixed workload (reload + prefill + Zipf decode, ms/step),
-the Llama-3-70B decode workload (GB/s), each with its own roofline, and the
+the Llama-3-70B decode workload (GB/s), each with its own roofline, the
 prefix-movement calibration (reload / offload bandwidth, the paper's
-mu / B_swap).
+mu / B_swap) and the redo trade of a preempted suffix (decode steps vs
+chunked prefill).
 
 Under torchrun every rank runs its own copy on its own GPU (the path has
 no exchange step: replicas only); value aggregates all ranks over the
@@ -336,6 +337,7 @@ def run_ours(args, rank, world, local_rank):
         result["decode_70b"] = bench_70b(args, dev, hbm_peak, peak_src)
         result["mixed"] = bench_mixed(args, dev)
         result["movement"] = bench_movement(args, dev)
+        result["redo"] = bench_redo(args, dev)
     if rank == 0 and world == 1 and not args.no_cpu:
         result["cpu_baseline"] = cpu_baseline(budget_s=15.0)
     return result
@@ -599,6 +601,76 @@ def bench_movement(args, dev):
     return res
 
 
+def bench_redo(args, dev):
+    """Rebuilding a preempted request's suffix KV (Sec. IV, Eq. 8 charges
+    T_decode y_r for redoing y_r tokens one decode step at a time) against
+    rebuilding it with chunked causal prefill (512-token chunks), both
+    through this library on one Llama-3-8B layer: one agent with a
+    4096-token prefix, one request whose suffix is rebuilt from empty."""
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+
+    hq, hkv, d, lp = 32, 8, 128, 4096
+    ys = [256, 1024, 4096]
+    ymax = max(ys)
+    ctx = B.allocate(num_q_heads=hq, num_kv_heads=hkv, head_dim=d,
+                     num_pages=(lp + ymax) // 16 + 64, max_agents=1, max_requests=1,
+                     max_tokens=512, max_seq_len=lp + ymax + 64, device=dev)
+    g = torch.Generator(device=dev).manual_seed(5)
+
+    def rnd(*shape):
+        return torch.randn(*shape, generator=g, device=dev).to(torch.bfloat16)
+    pk, pv = rnd(lp, hkv, d), rnd(lp, hkv, d)
+    q, k, v = rnd(ymax, hq, d), rnd(ymax, hkv, d), rnd(ymax, hkv, d)
+    out, lse = torch.empty(512, hq, d, dtype=torch.bfloat16, device=dev), \
+        torch.empty(512, hq, dtype=torch.float32, device=dev)
+    ctx.prefix_register(0, lp)
+    ctx.prefix_write(0, pk, pv)
+    ctx.request_open(0, 0)
+    one, zero = B.i32_array([0]), B.i32_array([0])
+    stream = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def run(fn):
+        ctx.request_truncate(one, zero)
+        fn()                                  # warm-up pass
+        torch.cuda.synchronize(dev)
+        ctx.request_truncate(one, zero)
+        ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+        ctx.kernel_times(reset=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        e1.synchronize()
+        kt = ctx.kernel_times(reset=True)
+        ctx.set_option(B.OPT_KERNEL_TIMING, 0)
+        return e0.elapsed_time(e1), sum(t for t, n in kt.values())
+
+    rows = []
+    for y in ys:
+        def by_decode():
+            for i in range(y):
+                ctx.decode(one, q[i:i + 1], k[i:i + 1], v[i:i + 1], out[:1], lse[:1], stream)
+
+        def by_prefill():
+            for o in range(0, y, 512):
+                c = min(512, y - o)
+                ctx.prefill_chunk(one, [c], q[o:o + c], k[o:o + c], v[o:o + c], out[:c], lse[:c],
+                                  stream)
+
+        wd, kd = run(by_decode)
+        wp, kp = run(by_prefill)
+        rows.append({"tokens": y, "decode_redo_ms": round(wd, 3), "decode_redo_kernel_ms": round(kd, 3),
+                     "prefill_rebuild_ms": round(wp, 3), "prefill_rebuild_kernel_ms": round(kp, 3),
+                     "T_decode_us_per_token": round(1e3 * kd / y, 2),
+                     "kernel_speedup": round(kd / kp, 1)})
+    st = ctx.device_status()
+    ctx.close()
+    return {"workload": "redo of a preempted request's suffix: llama3_8b layer, prefix 4096, "
+                        "suffix rebuilt from empty, decode (y steps) vs chunked prefill (512)",
+            "rows": rows, "device_status": st}
+
+
 # ------------------------------------------------------ oracle baseline --
 
 def _blas_threads():
@@ -700,7 +772,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement"],
+    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement", "redo"],
                     help="run just one of the extra workloads (1 GPU) and print its result")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -722,7 +794,8 @@ def main():
         fn = {"prefill": lambda: bench_prefill(args, dev, tf_peak, peak_src),
               "decode_70b": lambda: bench_70b(args, dev, hbm_peak, peak_src),
               "mixed": lambda: bench_mixed(args, dev),
-              "movement": lambda: bench_movement(args, dev)}[args.only]
+              "movement": lambda: bench_movement(args, dev),
+              "redo": lambda: bench_redo(args, dev)}[args.only]
         print(json.dumps({"only": args.only, "result": fn()}))
         return
     if world > 1:
