@@ -21,8 +21,9 @@ Also reported (rank 0, N=1): the tcgen05 chunked-prefill workload
 (TFLOP/s), the mixed workload (reload + prefill + Zipf decode, ms/step),
 the Llama-3-70B decode workload (GB/s), each with its own roofline, the
 prefix-movement calibration (reload / offload bandwidth, the paper's
-mu / B_swap) and the redo trade of a preempted suffix (decode steps vs
-chunked prefill).
+mu / B_swap), the redo trade of a preempted suffix (decode steps vs
+chunked prefill) and a kernel-level analogue of the paper's co-residency
+diagnostic (one vs two resident prefixes under one KV budget).
 
 Under torchrun every rank runs its own copy on its own GPU (the path has
 no exchange step: replicas only); value aggregates all ranks over the
@@ -338,6 +339,7 @@ def run_ours(args, rank, world, local_rank):
         result["mixed"] = bench_mixed(args, dev)
         result["movement"] = bench_movement(args, dev)
         result["redo"] = bench_redo(args, dev)
+        result["coresidency"] = bench_coresidency(args, dev)
     if rank == 0 and world == 1 and not args.no_cpu:
         result["cpu_baseline"] = cpu_baseline(budget_s=15.0)
     return result
@@ -671,6 +673,61 @@ def bench_redo(args, dev):
             "rows": rows, "device_status": st}
 
 
+def bench_coresidency(args, dev):
+    """Kernel-level analogue of the paper's Diagnostic 1 (Sec. II, Table 1):
+    under one KV budget, keeping one agent's long prefix resident (Grouped)
+    admits twice the decode batch of keeping two (Alternating).  Budget
+    49152 tokens of one Llama-3-8B layer; prefixes of 16384 tokens; each
+    request holds a 2048-token suffix.  Grouped: agent A resident, 16
+    requests; Alternating: A and B resident, 4 + 4 requests.  Each decode
+    step reads the whole budget either way; throughput follows the batch."""
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.session import Session
+    from paper_2608_25523_gb300.workloads import small_case, tensors_torch
+
+    lp, ls, budget = 16384, 2048, 49152
+    cases = {"grouped": ([lp], [0] * 16), "alternating": ([lp, lp], [0, 1] * 4)}
+    res = {"workload": f"KV budget {budget} tokens (llama3_8b layer), prefixes {lp}, "
+                       f"suffixes {ls}; decode steps of the admitted batch"}
+    stream = torch.cuda.current_stream(dev)
+    for name, (plens, agents) in cases.items():
+        n = len(agents)
+        assert sum(plens) + n * ls <= budget
+        w = small_case(7, hq=32, hkv=8, d=128, prefix_len=plens, req_agent=agents,
+                       req_ctx=[ls - 1] * n, req_prefill=[0] * n, req_decode=[1] * n)
+        t = tensors_torch(w, dev)
+        s = Session(w, t, device=dev, extra_tokens=16)
+        ids, q, kn, vn = s.decode_inputs()
+        out, lse = s.new_outputs(n)
+        ida, lna = B.i32_array(ids), B.i32_array([w.req_ctx[r] for r in ids])
+
+        def step():
+            s.ctx.decode(ida, q, kn, vn, out, lse, stream)
+            s.ctx.request_truncate(ida, lna)
+        for _ in range(10):
+            step()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        k = 200
+        e0.record(stream)
+        for _ in range(k):
+            step()
+        e1.record(stream)
+        e1.synchronize()
+        us = e0.elapsed_time(e1) / k * 1e3
+        step_bytes = decode_bytes(w, ids)[2]
+        res[name] = {"resident_prefixes": len(plens), "batch": n, "step_us": round(us, 2),
+                     "tokens_per_s": round(n / (us / 1e6), 1),
+                     "gbs": round(step_bytes / (us / 1e6) / 1e9, 1),
+                     "device_status": s.ctx.device_status()}
+        s.ctx.close()
+        del s, t
+    res["grouped_over_alternating_tokens_per_s"] = round(
+        res["grouped"]["tokens_per_s"] / res["alternating"]["tokens_per_s"], 2)
+    return res
+
+
 # ------------------------------------------------------ oracle baseline --
 
 def _blas_threads():
@@ -772,7 +829,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement", "redo"],
+    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement", "redo",
+                                       "coresidency"],
                     help="run just one of the extra workloads (1 GPU) and print its result")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -795,7 +853,8 @@ def main():
               "decode_70b": lambda: bench_70b(args, dev, hbm_peak, peak_src),
               "mixed": lambda: bench_mixed(args, dev),
               "movement": lambda: bench_movement(args, dev),
-              "redo": lambda: bench_redo(args, dev)}[args.only]
+              "redo": lambda: bench_redo(args, dev),
+              "coresidency": lambda: bench_coresidency(args, dev)}[args.only]
         print(json.dumps({"only": args.only, "result": fn()}))
         return
     if world > 1:
