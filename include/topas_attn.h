@@ -250,11 +250,16 @@ enum {
   TPA_OPT_PREFIX_SPLITS = 1,    /* cascade: key splits per stacked prefix tile; 0 = automatic */
   TPA_OPT_SUFFIX_SPLIT_KEYS = 2,/* keys per suffix work item, a multiple of 16; 0 = automatic */
   TPA_OPT_KERNEL_TIMING = 4,    /* 1: bracket every kernel with CUDA events (tpa_kernel_times) */
-  TPA_OPT_TEST_PLAN_WAIT = 5    /* test hook, 1: the next cascade decode's kernel waits for a
+  TPA_OPT_TEST_PLAN_WAIT = 5,   /* test hook, 1: the next cascade decode's kernel waits for a
                                    plan flag that is never written, so every CTA gives up at the
                                    device wait limit (2 s) without touching the pool and
                                    tpa_device_status reports TIMEOUT.  The context stays usable;
                                    truncate that call's requests back to their lengths before it */
+  TPA_OPT_PREFILL_TILE_ROWS = 6 /* query rows per prefill work item: 256 (default) pairs two
+                                   128-row tiles of 256/G consecutive tokens that share every K/V
+                                   tile (one CTA, two softmax warpgroups, the tensor pipe
+                                   alternating between them); 128 runs single tiles through the
+                                   dense kernel of the decode's level 1 */
 };
 TPA_API int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value);
 

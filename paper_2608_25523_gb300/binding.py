@@ -35,6 +35,7 @@ Q_LAST_DENSE_ITEMS, Q_LAST_SUFFIX_ITEMS, Q_LAST_LAUNCHES, Q_PAGE_OF = 5, 6, 7, 8
 OPT_DECODE_MODE, OPT_PREFIX_SPLITS, OPT_SUFFIX_SPLIT_KEYS = 0, 1, 2
 OPT_KERNEL_TIMING = 4
 OPT_TEST_PLAN_WAIT = 5
+OPT_PREFILL_TILE_ROWS = 6
 # kernel kinds of tpa_kernel_times
 KERNEL_NAMES = ["kv_append", "dense_tcgen05", "split_kv", "lse_merge", "page_copy"]
 

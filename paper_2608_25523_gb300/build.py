@@ -18,7 +18,7 @@ OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libtopas_attn.so")
 HEADER = os.path.join(ROOT, "include", "topas_attn.h")
 
-SOURCES = ["api.cu", "k_copy.cu", "k_merge.cu", "k_suffix.cu", "k_dense.cu", "no_alloc.cu"]
+SOURCES = ["api.cu", "k_copy.cu", "k_merge.cu", "k_suffix.cu", "k_dense.cu", "k_prefill.cu", "no_alloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden",
          "-I", os.path.join(ROOT, "include")]

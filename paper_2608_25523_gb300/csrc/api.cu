@@ -29,6 +29,7 @@
 namespace tpa {
 cudaError_t init_dense_kernels();
 cudaError_t init_suffix_kernels();
+cudaError_t init_prefill_pair();
 }  // namespace tpa
 
 using namespace tpa;
@@ -157,6 +158,7 @@ struct tpa_ctx {
 
   // options and statistics
   int decode_mode = 0;
+  int prefill_rows = 256;  // query rows per prefill work item: 256 (tile pairs) or 128
   int test_plan_wait = 0;  // test hook: the next cascade decode waits for a flag never written
   int prefix_splits = 0;
   int suffix_split_keys = 0;
@@ -1343,7 +1345,8 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   if (!ctx->plan_only && (!q || !k_new || !v_new || !out || !lse))
     return fail(TPA_ERR_INVALID_ARG, "null tensor");
   const int G = ctx->group, hkv = ctx->hkv;
-  const int tpt = kTileRows / G;
+  const bool pairs = ctx->prefill_rows == 2 * kTileRows;
+  const int tpt = (pairs ? 2 * kTileRows : kTileRows) / G;  // tokens per work item
 
   std::vector<int32_t> offset(n);
   for (int i = 0; i < n; ++i) offset[i] = ctx->reqs[reqs[i]].len;
@@ -1444,7 +1447,10 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
     DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
     dp.n_dense_ctas = std::min(nd, ctx->num_sms);
     KernelTimer kt(ctx, K_DENSE, s);
-    CUDA_TRY(launch_dense(dp, 0, ctx->d, G, false, s));
+    if (pairs)
+      CUDA_TRY(launch_prefill_pair(dp, dp.n_dense_ctas, ctx->d, G, s));
+    else
+      CUDA_TRY(launch_dense(dp, 0, ctx->d, G, false, s));
   }
   for (int i = 0; i < n; ++i) {
     Request& r = ctx->reqs[reqs[i]];
@@ -1575,6 +1581,10 @@ int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
     case TPA_OPT_TEST_PLAN_WAIT:
       ctx->test_plan_wait = value ? 1 : 0;
       return TPA_OK;
+    case TPA_OPT_PREFILL_TILE_ROWS:
+      if (value != 128 && value != 256) return fail(TPA_ERR_INVALID_ARG, "prefill tile rows %lld", (long long)value);
+      ctx->prefill_rows = static_cast<int>(value);
+      return TPA_OK;
     default: return fail(TPA_ERR_INVALID_ARG, "unknown option %d", option);
   }
 }
@@ -1618,6 +1628,8 @@ cudaError_t init_kernels() {
   cudaError_t e = init_dense_kernels();
   if (e != cudaSuccess) return e;
   e = init_suffix_kernels();
+  if (e != cudaSuccess) return e;
+  e = init_prefill_pair();
   if (e == cudaSuccess) done = true;
   return e;
 }

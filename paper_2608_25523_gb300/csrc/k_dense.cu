@@ -46,23 +46,19 @@
 // never a named barrier), drains its copies and MMAs, frees TMEM and returns.
 #include "kernels.h"
 #include "ptx.cuh"
+#include "dense_common.cuh"
 #include "split_kv.cuh"
 
 namespace tpa {
 
 namespace {
 
-constexpr float kLn2 = 0.6931471805599453f;
-constexpr float kRescaleThreshold = 8.0f;  // log2 units
+using namespace dense_detail;
+
+
 constexpr int kThreads = 352;               // K producer, MMA, 8 softmax warps, V producer
 constexpr int kWarpV = 10;                  // the V producer warp
 constexpr int kSoftmax = 256;
-
-__device__ __forceinline__ float fast_exp2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
 
 __device__ __forceinline__ void softmax_bar() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
 
@@ -97,32 +93,6 @@ struct DenseCfg {
 // barrier slots
 enum { B_KFULL = 0, B_KEMPTY = 3, B_VFULL = 6, B_VEMPTY = 9, B_SFULL = 12, B_SFREE = 14,
        B_PFULL = 16, B_PVDONE = 18, B_QFULL = 20, B_DRAIN = 21 };
-
-struct TileInfo {
-  int key0;     // first key of the tile within its segment
-  int nvalid;   // keys of the tile inside the range (1..128)
-  int causal;
-  int page_off; // page-list index of the tile's first page
-};
-
-__device__ __forceinline__ TileInfo tile_at(const DenseItem& it, int j) {
-  const int t0 = it.seg_k1[0] > it.seg_k0[0] ? (it.seg_k1[0] - it.seg_k0[0] + 127) / 128 : 0;
-  const int seg = j < t0 ? 0 : 1;
-  const int jj = j < t0 ? j : j - t0;
-  TileInfo t;
-  t.key0 = it.seg_k0[seg] + 128 * jj;
-  const int rest = it.seg_k1[seg] - t.key0;
-  t.nvalid = rest < 128 ? rest : 128;
-  t.causal = it.seg_causal[seg];
-  t.page_off = it.seg_pages[seg] + t.key0 / kPage;
-  return t;
-}
-
-// k-th item of this dense CTA: snake order over the dense CTAs on a
-// longest-first list.
-__device__ __forceinline__ int item_of(int k, int g) {
-  return k * g + ((k & 1) ? g - 1 - static_cast<int>(blockIdx.x) : static_cast<int>(blockIdx.x));
-}
 
 // Split-KV role of a CTA of the same launch: 8 independent warps, each with
 // a 3-stage TMA page ring in the shared memory the dense role would use.
@@ -223,109 +193,13 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   if (warp == 0 || warp == kWarpV) {
     // ------------------------------------------------------------ producers
     // Warp 0 streams K, warp kWarpV streams V, each through its own 3-stage
-    // ring, so K runs ahead of the PV pipeline.  Lane i (< 8) owns page i of
-    // every tile: it loads that page id ahead and issues the page's TMA box,
-    // so a tile's boxes go out from 8 lanes at once.  Lane 0 posts the
-    // expected byte count first.
+    // ring, so K runs ahead of the PV pipeline.
     const bool is_v = warp == kWarpV;
-    uint64_t* const full = bars + (is_v ? B_VFULL : B_KFULL);
-    uint64_t* const empty = bars + (is_v ? B_VEMPTY : B_KEMPTY);
-    const CUtensorMap* const tmap = is_v ? &p.tmap_v : &p.tmap_k;
-    uint8_t* const ring = smem + (is_v ? C::kOffV : C::kOffK);
-    int ph_last[C::kStages] = {-1, -1, -1};
-    bool pok = true;
-    auto wait_all = [&](uint64_t* bar, uint32_t parity) {
-      return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag)) != 0;
-    };
-    auto page_id = [&](const DenseItem& it, int j) -> int32_t {  // raw; validated when used
-      if (j >= it.n_tiles) return 0;
-      const TileInfo t = tile_at(it, j);
-      return lane < (t.nvalid + kPage - 1) / kPage ? __ldg(p.pages + t.page_off + lane) : 0;
-    };
-    // The current item and its first three tiles' page ids.  The next item's
-    // are loaded while the current one streams (the descriptor after tile 0
-    // is issued, the page ids after tile 1), so item boundaries add no load
-    // latency to the TMA stream.
-    DenseItem item{};
-    int32_t f0 = 0, f1 = 0, f2 = 0;
-    if (item_of(0, n_ctas) < p.n_items) {
-      item = p.items[item_of(0, n_ctas)];
-      f0 = page_id(item, 0);
-      f1 = page_id(item, 1);
-      f2 = page_id(item, 2);
-    }
-    int gt = 0;  // tiles of this CTA so far (ring position)
-    for (int k = 0; pok; ++k) {
-      const int idx = item_of(k, n_ctas);
-      if (idx >= p.n_items) break;
-      const int ntiles = item.n_tiles;
-      const int idx_n = item_of(k + 1, n_ctas);
-      const bool has_next = idx_n < p.n_items;
-      DenseItem nitem{};
-      int32_t n0 = 0, n1 = 0, n2 = 0;
-      bool next_ready = false;
-      // page ids loaded three tiles ahead
-      int32_t pid0 = f0, pid1 = f1, pid2 = f2;
-      for (int j = 0; j < ntiles; ++j, ++gt) {
-        const TileInfo t = tile_at(item, j);
-        const int s = gt % C::kStages;
-        const uint32_t ph = (gt / C::kStages) & 1;
-        const int npg = (t.nvalid + kPage - 1) / kPage;
-        const uint32_t bytes = static_cast<uint32_t>(npg * C::kPageBytes);
-        const int32_t pid = pid0;
-        pid0 = pid1;
-        pid1 = pid2;
-        pid2 = page_id(item, j + 3);
-        const bool bad = lane < npg && (pid < 0 || pid >= p.num_pages);
-        if (__any_sync(0xffffffffu, bad) && lane == 0 && !is_v) atomicOr(p.status, kStatusBadPage);
-        const int z = (bad ? 0 : pid) * p.hkv + item.kv_head;
-        // a full tile on 8 consecutive pages goes as one box of the kv head's
-        // page-run view; otherwise one box per page
-        const int32_t pid_0 = __shfl_sync(0xffffffffu, pid, 0);
-        const bool run = npg == 8 &&
-                         __all_sync(0xffffffffu, lane >= 8 || (!bad && pid == pid_0 + lane));
-        if (!wait_all(&empty[s], ph ^ 1u)) { pok = false; break; }
-        if (lane == 0) mbar_arrive_expect_tx(&full[s], bytes);
-        __syncwarp();
-        if (run) {
-          if (lane == 0)
-            tma_load_5d(ring + s * C::kKVBytes, p.run_maps + (is_v ? p.hkv : 0) + item.kv_head,
-                        &full[s], 0, 0, 0, 0, pid_0);
-        } else if (lane < npg) {
-          tma_load_5d(ring + s * C::kKVBytes + lane * C::kPageBytes, tmap, &full[s], 0, 0, 0, 0, z);
-        }
-        ph_last[s] = static_cast<int>(ph);
-        if (has_next && j == 0) nitem = p.items[idx_n];
-        if (has_next && j == 1) {
-          n0 = page_id(nitem, 0);
-          n1 = page_id(nitem, 1);
-          n2 = page_id(nitem, 2);
-          next_ready = true;
-        }
-      }
-      if (has_next && !next_ready) {
-        if (ntiles == 0) nitem = p.items[idx_n];
-        n0 = page_id(nitem, 0);
-        n1 = page_id(nitem, 1);
-        n2 = page_id(nitem, 2);
-      }
-      item = nitem;
-      f0 = n0;
-      f1 = n1;
-      f2 = n2;
-    }
-    if (!pok && lane == 0) {
-      *abort_flag = 1;
-      atomicOr(p.status, kStatusDenseTimeout);
-    }
-    __syncwarp();
-    if (*abort_flag && lane == 0) {
-      // let every issued copy land before the CTA's shared memory goes away
-      volatile int never = 0;
-      for (int s = 0; s < C::kStages; ++s)
-        if (ph_last[s] >= 0) (void)mbar_wait(&full[s], ph_last[s], &never);
-    }
-    __syncwarp();  // the warp reaches the teardown barrier converged
+    const bool pok = kv_producer<D, C::kStages>(
+        p, p.items, p.n_items, n_ctas, is_v ? &p.tmap_v : &p.tmap_k, p.run_maps + (is_v ? p.hkv : 0),
+        smem + (is_v ? C::kOffV : C::kOffK), bars + (is_v ? B_VFULL : B_KFULL),
+        bars + (is_v ? B_VEMPTY : B_KEMPTY), !is_v, abort_flag, lane);
+    if (!pok && lane == 0) atomicOr(p.status, kStatusDenseTimeout);
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {

@@ -77,6 +77,14 @@ struct DenseParams {
 cudaError_t launch_dense(const DenseParams& p, int n_split_ctas, int head_dim, int group,
                          bool dependent, cudaStream_t stream);
 
+// Chunked causal prefill, one persistent launch of `grid` CTAs (one per
+// SM) over items of two 128-row query tiles that share their key tiles
+// (tcgen05 + TMEM + TMA).  Items must have n_tok <= 256 / group and at
+// least one key tile; outputs go to p.out / p.lse (out_mode 1).  p.plan_flag
+// must be null.
+cudaError_t launch_prefill_pair(const DenseParams& p, int grid, int head_dim, int group,
+                                cudaStream_t stream);
+
 struct SuffixParams {
   CUtensorMap tmap_k;
   CUtensorMap tmap_v;

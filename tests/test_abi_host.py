@@ -206,10 +206,18 @@ def test_prefill_plan_decomposition(lib):
     ctx.prefix_register(1, 0)
     for r in range(4):
         ctx.request_open(r, r % 2)
+    # default: items of two 128-row tiles, 256/G tokens of one chunk
     ctx.prefill_chunk([0, 1, 2, 3], [512, 33, 1, 100], 1, 1, 1, 1, 1)
-    tiles_of = lambda c: math.ceil(c / (128 // G))
-    assert ctx.query(B.Q_LAST_DENSE_ITEMS) == hkv * sum(tiles_of(c) for c in (512, 33, 1, 100))
+    items_of = lambda c, rows: math.ceil(c / (rows // G))
+    assert ctx.query(B.Q_LAST_DENSE_ITEMS) == hkv * sum(items_of(c, 256) for c in (512, 33, 1, 100))
     assert [ctx.query(B.Q_SUFFIX_LEN, r) for r in range(4)] == [512, 33, 1, 100]
+    # single 128-row tiles
+    ctx.set_option(B.OPT_PREFILL_TILE_ROWS, 128)
+    ctx.prefill_chunk([0, 1, 2, 3], [64, 33, 1, 100], 1, 1, 1, 1, 1)
+    assert ctx.query(B.Q_LAST_DENSE_ITEMS) == hkv * sum(items_of(c, 128) for c in (64, 33, 1, 100))
+    assert [ctx.query(B.Q_SUFFIX_LEN, r) for r in range(4)] == [576, 66, 2, 200]
+    with pytest.raises(B.TpaError):
+        ctx.set_option(B.OPT_PREFILL_TILE_ROWS, 64)
 
 
 def test_permuted_pool_is_a_permutation(lib):

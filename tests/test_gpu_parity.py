@@ -131,17 +131,21 @@ PREFILL_CASES = {
     "d128_g4": (8, 2, 128, [0, 129, 1000], [0, 1, 2, 1, 2], [1, 31, 200, 64, 130], 64),
     "d64_g8": (16, 2, 64, [17, 128], [0, 1, 1], [33, 15, 150], 48),
     "d128_g8": (32, 4, 128, [250], [0, 0], [100, 17], 32),
+    # chunks of 100 tokens: pairs whose second tile holds 4, 5 and 18 tokens
+    "d128_g4_ragged_pairs": (8, 2, 128, [300, 0], [0, 1, 0], [100, 37, 250], 100),
 }
 
 
+@pytest.mark.parametrize("rows", [256, 128], ids=["pairs", "single"])
 @pytest.mark.parametrize("name", sorted(PREFILL_CASES))
-def test_prefill_chunks(name):
+def test_prefill_chunks(name, rows):
     hq, hkv, d, plen, agents, pf, chunk = PREFILL_CASES[name]
     n = len(agents)
     w = small_case(zlib.crc32(name.encode()) % 1000, hq=hq, hkv=hkv, d=d, prefix_len=plen, req_agent=agents,
                    req_ctx=[0] * n, req_prefill=pf, req_decode=[0] * n, chunk=chunk,
                    permute=True)
     t, s = _session(w)
+    s.ctx.set_option(B.OPT_PREFILL_TILE_ROWS, rows)
     for rnd in range(w.prefill_rounds()):
         chunks, ids, lens, q, k, v = s.prefill_inputs(rnd)
         out, lse = s.new_outputs(sum(lens))
