@@ -15,9 +15,10 @@
 //
 // A CTA owns one SM and walks its share of the items (longest first, snake
 // order):
-//   warps 0, 10 TMA producers of K (3-stage ring) and V (2-stage ring), as in
-//               the single-tile kernel (dense_common.cuh)
-//   warp 1      TMEM owner; one lane issues, in this fixed order per key
+//   warps 0..3  softmax of tile A, warps 4..7 of tile B (below)
+//   warps 8, 10 TMA producers of K (3-stage ring) and V (2-stage ring), as in
+//               the single-tile kernel (dense_common.cuh); warp 11 idles
+//   warp 9      TMEM owner; one lane issues, in this fixed order per key
 //               tile j (after S_A(0), S_B(0) of the item):
 //                 O_A += P_A(j) V_j,  S_A(j+1) = Q_A K_{j+1}^T,
 //                 O_B += P_B(j) V_j,  S_B(j+1) = Q_B K_{j+1}^T
@@ -25,8 +26,8 @@
 //               keys with P read from TMEM).  The tensor pipe runs a CTA's
 //               MMAs in issue order, so S_X(j+1) overwrites P_X(j) only after
 //               PV_X(j) has read it.
-//   warps 2..5  softmax of tile A, warps 6..9 of tile B: warp w owns TMEM
-//               lane quarter w % 4 and each thread one query row, all 128
+//   softmax     warp w owns TMEM lane quarter w % 4 and each thread one
+//               query row of its tile (a whole warpgroup per tile), all 128
 //               keys of a tile: read S, row max, P = 2^(s - m) as bf16 into
 //               the first 64 columns of its S buffer, row sum; O is rescaled
 //               in TMEM only when the max grew by more than 2^8 (the stale max
@@ -36,6 +37,9 @@
 //               the tile's last QK has completed.
 // TMEM (512 columns): S_A [0,128), S_B [128,256), O_A [256,256+d),
 // O_B [256+d,256+2d).
+// Registers: the launch gives every thread kLaunchRegs; the producer/MMA
+// warpgroup then drops to kLowRegs and the two softmax warpgroups rise to
+// kHighRegs (a whole S row, 128 floats, stays in registers), the same total.
 // Every mbarrier wait is bounded; on a timeout the CTA records a status bit,
 // every role stops, drains its copies and MMAs, frees TMEM and returns.
 #include "dense_common.cuh"
@@ -46,9 +50,13 @@ namespace {
 
 using namespace dense_detail;
 
-constexpr int kThreads = 352;  // K producer, MMA, 2 x 4 softmax warps, V producer
-constexpr int kWarpV = 10;
+constexpr int kThreads = 384;  // softmax warpgroups A and B, then K producer, MMA, V producer, idle
+constexpr int kWarpK = 8, kWarpMma = 9, kWarpV = 10;
 constexpr int kTileThreads = 128;  // softmax threads of one query tile
+constexpr int kLaunchRegs = 168;   // what ptxas assigns under __launch_bounds__(384, 1)
+constexpr int kLowRegs = 104, kHighRegs = 200;
+static_assert(2 * 128 * kHighRegs + 128 * kLowRegs == kThreads * kLaunchRegs,
+              "the register split redistributes exactly the launch allocation");
 
 template <int D>
 struct PairCfg {
@@ -118,13 +126,17 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
   }
   if (threadIdx.x >= 32 && threadIdx.x < 32 + 2 * p.hkv && p.run_maps)
     prefetch_tmap(p.run_maps + (threadIdx.x - 32));
-  if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
+  if (warp == kWarpMma) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0 || warp == kWarpV) {
+  // Each role's code sits inside the branch of its register change, so the
+  // compiler allocates it under that warpgroup's limit.
+  if (warp >= 8) {
+  setmaxnreg_dec<kLowRegs>();
+  if (warp == kWarpK || warp == kWarpV) {
     // ------------------------------------------------------------ producers
     const bool is_v = warp == kWarpV;
     bool pok;
@@ -137,7 +149,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
                                         smem + C::kOffK, bars + C::B_KFULL, bars + C::B_KEMPTY,
                                         true, abort_flag, lane);
     if (!pok && lane == 0) atomicOr(p.status, kStatusDenseTimeout);
-  } else if (warp == 1) {
+  } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc_qk = umma_idesc_bf16(128, 128, false, false);
@@ -225,9 +237,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
       (void)mbar_wait(&bars[C::B_DRAIN], 0, &never);
     }
     __syncwarp();
+  }
   } else {
+    setmaxnreg_inc<kHighRegs>();
     // ------------------------------------------------------------ softmax
-    const int x = (warp - 2) >> 2;           // query tile: 0 = A, 1 = B
+    const int x = warp >> 2;                 // query tile: 0 = A, 1 = B
     const int row = 32 * (warp & 3) + lane;  // row of the tile = TMEM lane
     const int tok_in = x * (128 / G) + row / G;  // token of the item
     const uint32_t lane_base = static_cast<uint32_t>(32 * (warp & 3)) << 16;
@@ -426,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
 
   // ---------------------------------------------------------------- teardown
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kWarpMma) {
     tc_fence_after();
     tmem_dealloc(tmem, C::kTmemCols);
   }
@@ -439,12 +453,27 @@ cudaError_t launch_prefill_pair_t(const DenseParams& p, int grid, cudaStream_t s
   return cudaGetLastError();
 }
 
+// Set once by init_prefill_pair: every instantiation was given kLaunchRegs
+// registers per thread, the allocation the warpgroup split redistributes.
+// With any other count an increase could wait forever, so the kernel is
+// not launched at all then.
+bool g_regs_checked = false;
+
+template <int D, int G>
+cudaError_t check_regs() {
+  cudaFuncAttributes a{};
+  cudaError_t e = cudaFuncGetAttributes(&a, prefill_pair_kernel<D, G>);
+  if (e != cudaSuccess) return e;
+  return a.numRegs == kLaunchRegs ? cudaSuccess : cudaErrorInvalidDeviceFunction;
+}
+
 }  // namespace
 
 cudaError_t launch_prefill_pair(const DenseParams& p, int grid, int head_dim, int group,
                                 cudaStream_t stream) {
   if (p.n_items <= 0 || grid <= 0) return cudaSuccess;
   if (p.plan_flag) return cudaErrorInvalidValue;  // the plan goes up on the launch stream
+  if (!g_regs_checked) return cudaErrorInvalidDeviceFunction;
   if (head_dim == 128 && group == 4) return launch_prefill_pair_t<128, 4>(p, grid, stream);
   if (head_dim == 128 && group == 8) return launch_prefill_pair_t<128, 8>(p, grid, stream);
   if (head_dim == 64 && group == 4) return launch_prefill_pair_t<64, 4>(p, grid, stream);
@@ -463,8 +492,14 @@ cudaError_t init_prefill_pair() {
   if ((e = cudaFuncSetAttribute(prefill_pair_kernel<64, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 PairCfg<64>::kSmem)))
     return e;
-  return cudaFuncSetAttribute(prefill_pair_kernel<64, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              PairCfg<64>::kSmem);
+  if ((e = cudaFuncSetAttribute(prefill_pair_kernel<64, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                PairCfg<64>::kSmem)))
+    return e;
+  // a wrong register count leaves the kernel unlaunchable (launches fail
+  // with cudaErrorInvalidDeviceFunction) without failing initialisation
+  g_regs_checked = check_regs<128, 4>() == cudaSuccess && check_regs<128, 8>() == cudaSuccess &&
+                   check_regs<64, 4>() == cudaSuccess && check_regs<64, 8>() == cudaSuccess;
+  return cudaSuccess;
 }
 
 }  // namespace tpa
