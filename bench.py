@@ -63,7 +63,7 @@ def peaks():
 
 # Sources of the unified decode kernel; the DRAM traffic recorded in its ncu
 # summary counts only while they are unchanged.
-KERNEL_SOURCES = ["k_dense.cu", "split_kv.cuh", "ptx.cuh", "plan.h", "kernels.h"]
+KERNEL_SOURCES = ["k_dense.cu", "dense_common.cuh", "split_kv.cuh", "ptx.cuh", "plan.h", "kernels.h"]
 PROFILE = os.path.join(ROOT, "profiles", "dense_tcgen05_c2_decode.md")
 
 
@@ -347,13 +347,16 @@ def run_ours(args, rank, world, local_rank):
 
 def bench_prefill(args, dev, tf_peak, peak_src):
     """Chunked causal prefill workload: all 512-token chunk rounds of 256
-    new requests over 8 agents' prefixes, timed as one pass."""
+    new requests over 8 agents' prefixes, timed as one pass (with
+    --prefill-stride k, every k-th request only: a small case of the same
+    shapes for profiler captures)."""
     import torch
     from paper_2608_25523_gb300 import binding as B
     from paper_2608_25523_gb300.session import Session
-    from paper_2608_25523_gb300.workloads import config, tensors_torch
+    from paper_2608_25523_gb300.workloads import config, request_subset, tensors_torch
 
-    w = config(2)
+    stride = max(1, getattr(args, "prefill_stride", 1))
+    w = config(2) if stride == 1 else request_subset(config(2), stride)
     stream = torch.cuda.current_stream(dev)
 
     def one_pass(kernel_timing=False):
@@ -382,16 +385,19 @@ def bench_prefill(args, dev, tf_peak, peak_src):
     _, kt, _, _ = one_pass(kernel_timing=True)
     flops = sum(prefill_flops(w, r[0]) for r in rounds)
     tokens = sum(sum(r[2]) for r in rounds)
-    dense_ms = kt["dense_tcgen05"][0]
+    kname = "prefill_pair_tcgen05"  # the default 256-row items
+    dense_ms = kt[kname][0]
     ach = flops / (dense_ms / 1e3) / 1e12
-    return {"workload": "chunked_prefill: 8 agents, prefixes U[2048,8192], 256 requests, suffixes "
-                        "U[512,2048] in 512-token chunks (all rounds)",
+    nreq = w.num_requests
+    return {"workload": f"chunked_prefill: 8 agents, prefixes U[2048,8192], {nreq} requests, suffixes "
+                        "U[512,2048] in 512-token chunks (all rounds)" +
+                        (f", every {stride}th request of the 256" if stride > 1 else ""),
             "tflops": round(flops / (ms / 1e3) / 1e12, 1), "ms": round(ms, 3),
             "tokens_per_s": round(tokens / (ms / 1e3), 1), "flops": flops,
-            "roofline": {"bound": "tensor", "kernel": "dense_tcgen05", "achieved": round(ach, 1),
+            "roofline": {"bound": "tensor", "kernel": kname, "achieved": round(ach, 1),
                          "peak": tf_peak, "unit": "TFLOP/s", "frac": round(ach / tf_peak, 4),
                          "peak_source": peak_src, "traffic": None,
-                         "avg_launch_us": round(1e3 * dense_ms / max(1, kt["dense_tcgen05"][1]), 1)},
+                         "avg_launch_us": round(1e3 * dense_ms / max(1, kt[kname][1]), 1)},
             "device_status": st}
 
 
@@ -832,6 +838,8 @@ def main():
     ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement", "redo",
                                        "coresidency"],
                     help="run just one of the extra workloads (1 GPU) and print its result")
+    ap.add_argument("--prefill-stride", type=int, default=1,
+                    help="prefill workload: every k-th request only (a small case for profiling)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     rank = int(os.environ.get("RANK", 0))

@@ -267,7 +267,8 @@ TPA_API int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value);
  * every kernel launch of the library is bracketed by CUDA events on the
  * stream it runs on.  This call synchronises with those events and returns,
  * for each kernel kind k < n (0 KV append, 1 dense tensor-core attention,
- * 2 split-KV attention, 3 LSE merge, 4 page-run copy), the accumulated time
+ * 2 split-KV attention, 3 LSE merge, 4 page-run copy, 5 paired-tile
+ * tensor-core prefill), the accumulated time
  * in milliseconds and the number of launches since the last reset
  * (`reset` != 0 clears the totals after reading).  Errors: INVALID_ARG, CUDA. */
 TPA_API int tpa_kernel_times(tpa_ctx* ctx, int32_t n, double* total_ms, int64_t* launches,

@@ -37,7 +37,8 @@ OPT_KERNEL_TIMING = 4
 OPT_TEST_PLAN_WAIT = 5
 OPT_PREFILL_TILE_ROWS = 6
 # kernel kinds of tpa_kernel_times
-KERNEL_NAMES = ["kv_append", "dense_tcgen05", "split_kv", "lse_merge", "page_copy"]
+KERNEL_NAMES = ["kv_append", "dense_tcgen05", "split_kv", "lse_merge", "page_copy",
+                "prefill_pair_tcgen05"]
 
 
 class TpaError(RuntimeError):

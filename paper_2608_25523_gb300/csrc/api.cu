@@ -58,8 +58,8 @@ int fail(int code, const char* fmt, ...) {
 
 constexpr int kRingSlots = 4;
 constexpr int kSplitWarpsPerCta = 8;  // split-KV warps of a CTA in the fused decode launch
-constexpr int kKernelKinds = 5;  // append, dense, split-KV, merge, page copy
-enum { K_APPEND = 0, K_DENSE = 1, K_SUFFIX = 2, K_MERGE = 3, K_COPY = 4 };
+constexpr int kKernelKinds = 6;  // append, dense, split-KV, merge, page copy, paired prefill
+enum { K_APPEND = 0, K_DENSE = 1, K_SUFFIX = 2, K_MERGE = 3, K_COPY = 4, K_PREFILL_PAIR = 5 };
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -1446,7 +1446,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
     }
     DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
     dp.n_dense_ctas = std::min(nd, ctx->num_sms);
-    KernelTimer kt(ctx, K_DENSE, s);
+    KernelTimer kt(ctx, pairs ? K_PREFILL_PAIR : K_DENSE, s);
     if (pairs)
       CUDA_TRY(launch_prefill_pair(dp, dp.n_dense_ctas, ctx->d, G, s));
     else

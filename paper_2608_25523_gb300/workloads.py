@@ -281,6 +281,19 @@ def replicate(w: Workload, copies: int) -> Workload:
         reload_agents=[a + c * na for c in range(copies) for a in w.reload_agents])
 
 
+def request_subset(w: Workload, stride: int) -> Workload:
+    """Every `stride`-th request of a workload (all its agents kept): the
+    same shapes and prefixes with fewer new tokens, for profiler captures
+    that must hold little device memory."""
+    keep = list(range(0, w.num_requests, stride))
+    return replace(
+        w, name=f"{w.name}_every{stride}",
+        req_agent=[w.req_agent[r] for r in keep],
+        req_ctx=[w.req_ctx[r] for r in keep],
+        req_prefill=[w.req_prefill[r] for r in keep],
+        req_decode=[w.req_decode[r] for r in keep])
+
+
 def copy_requests(w: Workload, copies: int, c: int) -> list:
     """Request ids of copy `c` of replicate(w, copies)."""
     n = w.num_requests // copies
