@@ -16,7 +16,8 @@ value  = algorithmic bytes per step (each prefix once, each suffix once,
          Q, the new tokens' K/V in and out, O and LSE) / device time, GB/s.
 e2e    = the same metric through the public call with host buffers: the
          step's q / k_new / v_new come from pinned host memory and O / LSE
-         go back, inside the timed region.
+         go back, inside the timed region (each packed in one buffer: one
+         copy each way per step).
 Also reported (rank 0, N=1): the tcgen05 chunked-prefill workload
 (TFLOP/s), the mixed workload (reload + prefill + Zipf decode, ms/step),
 the Llama-3-70B decode workload (GB/s), each with its own roofline, the
@@ -270,25 +271,40 @@ def run_ours(args, rank, world, local_rank):
 
     # end to end through the public call with host buffers
     import torch as _t
-    host = []
+    # A step's inputs (q, k_new, v_new) sit back to back in one pinned host
+    # buffer and one device buffer, and so do its outputs (out, lse): one
+    # host-to-device and one device-to-host copy per step.
+    def packed(tensors, device):
+        sizes = [x.numel() * x.element_size() for x in tensors]
+        buf = _t.empty(sum(sizes), dtype=_t.uint8, device=device,
+                       pin_memory=device == "cpu")
+        views, off = [], 0
+        for x, n in zip(tensors, sizes):
+            views.append(buf[off:off + n].view(x.dtype).view(x.shape))
+            off += n
+        return buf, views
+
+    host, dev_io = [], []
     for ids, q, kn, vn, out, lse, lens in steps:
-        hq, hk, hv = (x.cpu().pin_memory() for x in (q, kn, vn))
-        ho = _t.empty(out.shape, dtype=out.dtype, pin_memory=True)
-        hl = _t.empty(lse.shape, dtype=lse.dtype, pin_memory=True)
-        host.append((hq, hk, hv, ho, hl))
-    h2d = sum(x.numel() * x.element_size() for x in host[0][:3])
-    d2h = sum(x.numel() * x.element_size() for x in host[0][3:])
+        hin, hviews = packed((q, kn, vn), "cpu")
+        for hv_, x in zip(hviews, (q, kn, vn)):
+            hv_.copy_(x.cpu())
+        hout, _ = packed((out, lse), "cpu")
+        din, (dq, dkn, dvn) = packed((q, kn, vn), dev)
+        dout, (dou, dls) = packed((out, lse), dev)
+        host.append((hin, hout))
+        dev_io.append((din, dq, dkn, dvn, dout, dou, dls))
+    h2d = host[0][0].numel()
+    d2h = host[0][1].numel()
     e2e_steps = args.steps
 
     def e2e_step(i):
-        ids, q, kn, vn, out, lse, lens = steps[i % COPIES]
-        hq, hk, hv, ho, hl = host[i % COPIES]
-        q.copy_(hq, non_blocking=True)
-        kn.copy_(hk, non_blocking=True)
-        vn.copy_(hv, non_blocking=True)
-        s.ctx.decode(ids, q, kn, vn, out, lse, stream)
-        ho.copy_(out, non_blocking=True)
-        hl.copy_(lse, non_blocking=True)
+        ids, _, _, _, _, _, lens = steps[i % COPIES]
+        hin, hout = host[i % COPIES]
+        din, dq, dkn, dvn, dout, dou, dls = dev_io[i % COPIES]
+        din.copy_(hin, non_blocking=True)
+        s.ctx.decode(ids, dq, dkn, dvn, dou, dls, stream)
+        hout.copy_(dout, non_blocking=True)
         s.ctx.request_truncate(ids, lens)
 
     for i in range(args.warmup):
