@@ -53,6 +53,8 @@ does):
       active agents A_t (a resident prefix without requests cannot be
       covered, so it always leaves); repairs drop one agent of R or swap
       one for an agent of A_t outside R.
+  R10 When no state is generated at all (the caps forbid every change and
+      the incumbent's requests do not all fit), the incumbent is kept.
 """
 from __future__ import annotations
 
@@ -393,6 +395,9 @@ def decide(s: Snapshot, p: Params) -> State:
         # the incumbent itself
         inc_keep = [r for r in range(nreq) if s.req_running[r]]
         cands.append(score_state(s, p, r_now, inc_keep, [], [], n_a))
+    if not cands:   # R10
+        cands.append(score_state(s, p, r_now, [r for r in range(nreq) if s.req_running[r]],
+                                 [], [], n_a))
     nonempty = [st for st in cands if st.running]
     if nonempty:
         cands = nonempty

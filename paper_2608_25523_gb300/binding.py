@@ -1,4 +1,4 @@
-"""ctypes binding of libtopas_attn.so (include/topas_attn.h).
+"""ctypes binding of libtopas_attn.so (include/topas_attn.h, include/topas_sched.h).
 
 Argument marshalling only: every step of the attention path runs in the
 library's CUDA kernels.  Loading fails loudly when the library has not been
@@ -9,9 +9,10 @@ from __future__ import annotations
 import ctypes
 import os
 import re
-from ctypes import POINTER, c_char_p, c_int, c_int32, c_int64, c_size_t, c_uint32, c_uint64, c_void_p
+from ctypes import (POINTER, c_char_p, c_double, c_int, c_int8, c_int32, c_int64, c_size_t, c_uint8,
+                    c_uint32, c_uint64, c_void_p)
 
-from .build import HEADER, LIB
+from .build import HEADER, LIB, SCHED_HEADER
 
 # status codes
 TPA_OK = 0
@@ -57,6 +58,33 @@ class Config(ctypes.Structure):
 
 
 _I32P = POINTER(c_int32)
+class SchedParams(ctypes.Structure):
+    _fields_ = [("budget", c_double), ("mu", c_double), ("b_swap", c_double), ("t_decode", c_double),
+                ("beta", c_double), ("rho", c_double), ("h_age", c_double), ("M", c_int32),
+                ("K", c_int32), ("mc_samples", c_int32), ("pad", c_int32), ("seed", c_uint64)]
+
+
+class SchedSnapshot(ctypes.Structure):
+    _fields_ = [("t", c_double), ("n_stages", c_int32), ("n_agents", c_int32), ("n_tasks", c_int32),
+                ("n_reqs", c_int32), ("stage_agent", POINTER(c_int32)), ("pred_off", POINTER(c_int32)),
+                ("pred_idx", POINTER(c_int32)), ("prefix_len", POINTER(c_int64)),
+                ("sample_off", POINTER(c_int32)), ("samples", POINTER(c_double)),
+                ("task_id", POINTER(c_uint64)), ("task_arrival", POINTER(c_double)),
+                ("stage_state", POINTER(c_int8)), ("stage_served", POINTER(c_double)),
+                ("req_task", POINTER(c_int32)), ("req_stage", POINTER(c_int32)),
+                ("req_kv", POINTER(c_double)), ("req_dhat", POINTER(c_double)),
+                ("req_redo", POINTER(c_double)), ("req_credit", POINTER(c_double)),
+                ("req_running", POINTER(c_uint8)), ("resident", POINTER(c_uint8))]
+
+
+class SchedDecision(ctypes.Structure):
+    _fields_ = [("agents", POINTER(c_uint8)), ("running", POINTER(c_uint8)),
+                ("admitted", POINTER(c_int32)), ("credits", POINTER(c_double)),
+                ("n_admitted", c_int32), ("n_preempted", c_int32), ("score", c_double),
+                ("j_admit", c_double), ("j_move", c_double), ("j_redo", c_double),
+                ("j_revoke", c_double), ("v_reuse", c_double), ("n_candidates", c_int64)]
+
+
 _SIGS = {
     "tpa_workspace_size": (c_size_t, [POINTER(Config)]),
     "tpa_create": (c_int, [POINTER(Config), POINTER(c_void_p)]),
@@ -83,14 +111,15 @@ _SIGS = {
     "tpa_kernel_times": (c_int, [c_void_p, c_int32, POINTER(ctypes.c_double), POINTER(c_int64),
                                  c_int32]),
     "tpa_last_error": (c_char_p, []),
+    "tpa_sched_decide": (c_int, [POINTER(SchedParams), POINTER(SchedSnapshot), POINTER(SchedDecision)]),
 }
 
 _lib = None
 
 
 def header_functions() -> list:
-    """Names of the functions include/topas_attn.h declares."""
-    text = open(HEADER).read()
+    """Names of the functions include/topas_attn.h and include/topas_sched.h declare."""
+    text = open(HEADER).read() + open(SCHED_HEADER).read()
     return sorted(set(re.findall(r"^TPA_API\s+[\w\s\*]+?\b(tpa_\w+)\s*\(", text, re.M)))
 
 
@@ -293,3 +322,63 @@ def allocate(*, num_q_heads, num_kv_heads, head_dim, num_pages, max_agents, max_
     ctx = Context(cfg, keep=(k_pool, v_pool, ws))
     ctx.k_pool, ctx.v_pool, ctx.workspace = k_pool, v_pool, ws
     return ctx
+
+
+# ---------------------------------------------------------------- scheduler
+
+def _arr(ctype, vals):
+    vals = list(vals)
+    return (ctype * max(1, len(vals)))(*vals)
+
+
+def sched_decide(params, snap) -> dict:
+    """tpa_sched_decide (include/topas_sched.h).
+
+    `params` and `snap` are any objects with the header's field names, the
+    snapshot's per-stage predecessors and samples as `stage_preds` and
+    `stage_samples` (lists of lists) and its [task][stage] arrays as lists of
+    lists.  Returns the selected state: R' and Q' (sorted ids), the admitted
+    requests in order with their credits, the preempted count and the score
+    terms of Eq. 12."""
+    lib = load()
+    ns, na, nt, nr = (len(snap.stage_agent), len(snap.prefix_len), len(snap.task_id),
+                      len(snap.req_task))
+    pred_off, pred_idx = [0], []
+    for preds in snap.stage_preds:
+        pred_idx += list(preds)
+        pred_off.append(len(pred_idx))
+    sample_off, samples = [0], []
+    for xs in snap.stage_samples:
+        samples += list(xs)
+        sample_off.append(len(samples))
+    keep = dict(
+        stage_agent=_arr(c_int32, snap.stage_agent), pred_off=_arr(c_int32, pred_off),
+        pred_idx=_arr(c_int32, pred_idx), prefix_len=_arr(c_int64, snap.prefix_len),
+        sample_off=_arr(c_int32, sample_off), samples=_arr(c_double, samples),
+        task_id=_arr(c_uint64, snap.task_id), task_arrival=_arr(c_double, snap.task_arrival),
+        stage_state=_arr(c_int8, [x for row in snap.stage_state for x in row]),
+        stage_served=_arr(c_double, [x for row in snap.stage_served for x in row]),
+        req_task=_arr(c_int32, snap.req_task), req_stage=_arr(c_int32, snap.req_stage),
+        req_kv=_arr(c_double, snap.req_kv), req_dhat=_arr(c_double, snap.req_dhat),
+        req_redo=_arr(c_double, snap.req_redo), req_credit=_arr(c_double, snap.req_credit),
+        req_running=_arr(c_uint8, [1 if x else 0 for x in snap.req_running]),
+        resident=_arr(c_uint8, [1 if x else 0 for x in snap.resident]))
+    cs = SchedSnapshot(snap.t, ns, na, nt, nr,
+                       *(ctypes.cast(keep[f], ptype) for f, ptype in SchedSnapshot._fields_[5:]))
+    cp = SchedParams(params.budget, params.mu, params.b_swap, params.t_decode, params.beta,
+                     params.rho, params.h_age, params.M, params.K, params.mc_samples, 0,
+                     params.seed)
+    out_agents, out_running = (c_uint8 * na)(), (c_uint8 * max(1, nr))()
+    out_adm, out_cred = (c_int32 * max(1, nr))(), (c_double * max(1, nr))()
+    cd = SchedDecision(out_agents, out_running, out_adm, out_cred)
+    rc = lib.tpa_sched_decide(ctypes.byref(cp), ctypes.byref(cs), ctypes.byref(cd))
+    if rc != TPA_OK:
+        raise TpaError(rc, lib.tpa_last_error().decode())
+    n = cd.n_admitted
+    return {"agents": tuple(a for a in range(na) if out_agents[a]),
+            "running": tuple(r for r in range(nr) if out_running[r]),
+            "admitted": tuple(out_adm[k] for k in range(n)),
+            "credits": tuple(out_cred[k] for k in range(n)),
+            "n_preempted": cd.n_preempted, "score": cd.score, "j_admit": cd.j_admit,
+            "j_move": cd.j_move, "j_redo": cd.j_redo, "j_revoke": cd.j_revoke,
+            "v_reuse": cd.v_reuse, "n_candidates": cd.n_candidates}

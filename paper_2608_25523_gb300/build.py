@@ -17,8 +17,13 @@ CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libtopas_attn.so")
 HEADER = os.path.join(ROOT, "include", "topas_attn.h")
+SCHED_HEADER = os.path.join(ROOT, "include", "topas_sched.h")
 
-SOURCES = ["api.cu", "k_copy.cu", "k_merge.cu", "k_suffix.cu", "k_dense.cu", "k_prefill.cu", "no_alloc.cu"]
+SOURCES = ["api.cu", "k_copy.cu", "k_merge.cu", "k_suffix.cu", "k_dense.cu", "k_prefill.cu", "no_alloc.cu",
+           "sched.cpp"]
+# per-file flags: the scheduler's fp64 arithmetic must not be contracted into
+# FMAs (its decisions are compared with a plain restatement bit for bit)
+EXTRA = {"sched.cpp": ["-Xcompiler", "-ffp-contract=off"]}
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden",
          "-I", os.path.join(ROOT, "include")]
@@ -32,18 +37,18 @@ def _nvcc() -> str:
 
 
 def _deps_mtime() -> float:
-    files = [HEADER] + [os.path.join(CSRC, f) for f in os.listdir(CSRC)
-                        if f.endswith((".h", ".cuh"))]
+    files = [HEADER, SCHED_HEADER] + [
+        os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
     return max(os.path.getmtime(f) for f in files)
 
 
 def _compile(nvcc: str, src: str, verbose: bool) -> str:
-    obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
+    obj = os.path.join(OUT_DIR, os.path.splitext(src)[0] + ".o")
     path = os.path.join(CSRC, src)
     if (os.path.exists(obj) and os.path.getmtime(obj) >= os.path.getmtime(path)
             and os.path.getmtime(obj) >= _deps_mtime()):
         return obj
-    cmd = [nvcc, *ARCH, *FLAGS, "-c", path, "-o", obj]
+    cmd = [nvcc, *ARCH, *FLAGS, *EXTRA.get(src, []), "-c", path, "-o", obj]
     if verbose:
         cmd.insert(1, "-Xptxas=-v")
     res = subprocess.run(cmd, capture_output=True, text=True)

@@ -1622,6 +1622,8 @@ int tpa_device_status(tpa_ctx* ctx, void* stream, uint32_t* status) {
 }  // extern "C"
 
 namespace tpa {
+int set_error(int code, const char* msg) { return fail(code, "%s", msg); }
+
 cudaError_t init_kernels() {
   static bool done = false;
   if (done) return cudaSuccess;
