@@ -23,8 +23,10 @@ Also reported (rank 0, N=1): the tcgen05 chunked-prefill workload
 the Llama-3-70B decode workload (GB/s), each with its own roofline, the
 prefix-movement calibration (reload / offload bandwidth, the paper's
 mu / B_swap), the redo trade of a preempted suffix (decode steps vs
-chunked prefill) and a kernel-level analogue of the paper's co-residency
-diagnostic (one vs two resident prefixes under one KV budget).
+chunked prefill), a kernel-level analogue of the paper's co-residency
+diagnostic (one vs two resident prefixes under one KV budget), and the
+TOPAS scheduler driving the library on Chain-3 tasks (decision latency,
+native and oracle).
 
 Under torchrun every rank runs its own copy on its own GPU (the path has
 no exchange step: replicas only); value aggregates all ranks over the
@@ -356,6 +358,7 @@ def run_ours(args, rank, world, local_rank):
         result["movement"] = bench_movement(args, dev)
         result["redo"] = bench_redo(args, dev)
         result["coresidency"] = bench_coresidency(args, dev)
+        result["sched"] = bench_sched(args, dev)
     if rank == 0 and world == 1 and not args.no_cpu:
         result["cpu_baseline"] = cpu_baseline(budget_s=15.0)
     return result
@@ -415,6 +418,56 @@ def bench_prefill(args, dev, tf_peak, peak_src):
                          "peak_source": peak_src, "traffic": None,
                          "avg_launch_us": round(1e3 * dense_ms / max(1, kt[kname][1]), 1)},
             "device_status": st}
+
+
+def bench_sched(args, dev):
+    """TOPAS decisions driving the library (the scheduler of Sec. IV as a host
+    module): Chain-3 tasks on the Llama-3-8B attention layer under a KV budget
+    that forces prefix moves and preemptions.  Service times are synthetic;
+    the page table and the attention kernels are real.  Reports the native
+    decision latency and, as its CPU baseline, the oracle's on the same
+    recorded snapshots."""
+    import time
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.workflow_sim import WorkflowSim, chain3
+
+    wf = chain3()
+    pages = 900     # the three prefixes need 576 pages: room for a few requests
+    ctx = B.allocate(num_q_heads=32, num_kv_heads=8, head_dim=128, num_pages=pages, max_agents=8,
+                     max_requests=64, max_tokens=1024, max_seq_len=8192, device=str(dev))
+    ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+    rec = []
+    sim = WorkflowSim(wf, ctx, n_tasks=40, rate=1.5, seed=7, dims=(32, 8, 128), budget_pages=pages,
+                      max_tokens=1024, max_requests=64, device=str(dev), record=rec)
+    res = sim.run()
+    torch.cuda.synchronize(dev)
+    kt = ctx.kernel_times(reset=True)
+    st = ctx.device_status()
+    ctx.close()
+    native = [B.sched_decide(prm, snap, repeat=20)["native_us"] for prm, snap, _ in rec]
+    out = res.summary()
+    out.update({
+        "workload": "chain3 workflow (3 agents, prefixes 2048/4096/3072 tokens), 40 tasks, "
+                    "Poisson 1.5/s, KV budget 900 pages; Llama-3-8B layer (Hq 32, Hkv 8, d 128); "
+                    "synthetic service times (20 us/prefill token, 20 ms/decode step)",
+        "native_decide_us_mean": round(sum(native) / len(native), 1),
+        "native_decide_us_max": round(max(native), 1),
+        "gpu_ms": {k: round(v[0], 3) for k, v in kt.items() if v[1]},
+        "device_status": st})
+    if not args.no_cpu:
+        import oracle.sched as OS   # CPU baseline: the oracle on the same snapshots
+        t0 = time.perf_counter()
+        n = 0
+        for prm, snap, _ in rec:
+            OS.decide(OS.Snapshot(**vars(snap)), OS.Params(**vars(prm)))
+            n += 1
+            if time.perf_counter() - t0 > 10.0:
+                break
+        out["cpu_baseline"] = {"value": round((time.perf_counter() - t0) / n * 1e6, 1), "unit": "us/decision",
+                               "cores": 1, "kind": "oracle",
+                               "sample": f"the first {n} of {len(rec)} recorded decisions"}
+    return out
 
 
 def bench_70b(args, dev, hbm_peak, peak_src):
@@ -852,7 +905,7 @@ def main():
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement", "redo",
-                                       "coresidency"],
+                                       "coresidency", "sched"],
                     help="run just one of the extra workloads (1 GPU) and print its result")
     ap.add_argument("--prefill-stride", type=int, default=1,
                     help="prefill workload: every k-th request only (a small case for profiling)")
@@ -878,7 +931,8 @@ def main():
               "mixed": lambda: bench_mixed(args, dev),
               "movement": lambda: bench_movement(args, dev),
               "redo": lambda: bench_redo(args, dev),
-              "coresidency": lambda: bench_coresidency(args, dev)}[args.only]
+              "coresidency": lambda: bench_coresidency(args, dev),
+              "sched": lambda: bench_sched(args, dev)}[args.only]
         print(json.dumps({"only": args.only, "result": fn()}))
         return
     if world > 1:

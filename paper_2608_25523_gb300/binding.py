@@ -331,7 +331,7 @@ def _arr(ctype, vals):
     return (ctype * max(1, len(vals)))(*vals)
 
 
-def sched_decide(params, snap) -> dict:
+def sched_decide(params, snap, repeat: int = 1) -> dict:
     """tpa_sched_decide (include/topas_sched.h).
 
     `params` and `snap` are any objects with the header's field names, the
@@ -339,7 +339,9 @@ def sched_decide(params, snap) -> dict:
     `stage_samples` (lists of lists) and its [task][stage] arrays as lists of
     lists.  Returns the selected state: R' and Q' (sorted ids), the admitted
     requests in order with their credits, the preempted count and the score
-    terms of Eq. 12."""
+    terms of Eq. 12.  With repeat > 1 the native call runs that many times
+    on the marshalled arguments and `native_us` is its mean duration."""
+    import time
     lib = load()
     ns, na, nt, nr = (len(snap.stage_agent), len(snap.prefix_len), len(snap.task_id),
                       len(snap.req_task))
@@ -371,9 +373,12 @@ def sched_decide(params, snap) -> dict:
     out_agents, out_running = (c_uint8 * na)(), (c_uint8 * max(1, nr))()
     out_adm, out_cred = (c_int32 * max(1, nr))(), (c_double * max(1, nr))()
     cd = SchedDecision(out_agents, out_running, out_adm, out_cred)
-    rc = lib.tpa_sched_decide(ctypes.byref(cp), ctypes.byref(cs), ctypes.byref(cd))
-    if rc != TPA_OK:
-        raise TpaError(rc, lib.tpa_last_error().decode())
+    t0 = time.perf_counter()
+    for _ in range(max(1, repeat)):
+        rc = lib.tpa_sched_decide(ctypes.byref(cp), ctypes.byref(cs), ctypes.byref(cd))
+        if rc != TPA_OK:
+            raise TpaError(rc, lib.tpa_last_error().decode())
+    native_us = (time.perf_counter() - t0) / max(1, repeat) * 1e6
     n = cd.n_admitted
     return {"agents": tuple(a for a in range(na) if out_agents[a]),
             "running": tuple(r for r in range(nr) if out_running[r]),
@@ -381,4 +386,4 @@ def sched_decide(params, snap) -> dict:
             "credits": tuple(out_cred[k] for k in range(n)),
             "n_preempted": cd.n_preempted, "score": cd.score, "j_admit": cd.j_admit,
             "j_move": cd.j_move, "j_redo": cd.j_redo, "j_revoke": cd.j_revoke,
-            "v_reuse": cd.v_reuse, "n_candidates": cd.n_candidates}
+            "v_reuse": cd.v_reuse, "n_candidates": cd.n_candidates, "native_us": native_us}
