@@ -255,7 +255,12 @@ enum {
                                    device wait limit (2 s) without touching the pool and
                                    tpa_device_status reports TIMEOUT.  The context stays usable;
                                    truncate that call's requests back to their lengths before it */
-  TPA_OPT_PREFILL_TILE_ROWS = 6 /* query rows per prefill work item: 256 (default) pairs two
+  TPA_OPT_TEST_BAD_PAGE = 7,    /* test hook, 1: the next decode's plan lists its first resident
+                                   prefix's first page as the pool size (one past the last page).
+                                   Every kernel bounds-checks page ids: those reads go to page 0 and
+                                   the device status gets bit 4; that step's outputs for the agent's
+                                   tokens are wrong, and later steps are unaffected */
+  TPA_OPT_PREFILL_TILE_ROWS = 6,/* query rows per prefill work item: 256 (default) pairs two
                                    128-row tiles of 256/G consecutive tokens that share every K/V
                                    tile (one CTA, two softmax warpgroups, the tensor pipe
                                    alternating between them); 128 runs single tiles through the

@@ -37,6 +37,7 @@ OPT_DECODE_MODE, OPT_PREFIX_SPLITS, OPT_SUFFIX_SPLIT_KEYS = 0, 1, 2
 OPT_KERNEL_TIMING = 4
 OPT_TEST_PLAN_WAIT = 5
 OPT_PREFILL_TILE_ROWS = 6
+OPT_TEST_BAD_PAGE = 7
 # kernel kinds of tpa_kernel_times
 KERNEL_NAMES = ["kv_append", "dense_tcgen05", "split_kv", "lse_merge", "page_copy",
                 "prefill_pair_tcgen05"]

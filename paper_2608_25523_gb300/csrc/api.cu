@@ -160,6 +160,7 @@ struct tpa_ctx {
   int decode_mode = 0;
   int prefill_rows = 256;  // query rows per prefill work item: 256 (tile pairs) or 128
   int test_plan_wait = 0;  // test hook: the next cascade decode waits for a flag never written
+  int test_bad_page = 0;   // test hook: the next decode's first prefix page id is out of the pool
   int prefix_splits = 0;
   int suffix_split_keys = 0;
   int64_t last_dense = 0, last_suffix = 0, last_launches = 0;
@@ -1141,6 +1142,11 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     std::memcpy(w.pages + np, a.pages.data(), a.pages.size() * 4);
     np += static_cast<int32_t>(a.pages.size());
   }
+  if (ctx->test_bad_page && !groups.empty() && !ctx->agents[groups[0].agent].pages.empty()) {
+    // a read-only prefix page: every kernel read of it is bounds-checked
+    w.pages[0] = static_cast<int32_t>(ctx->cfg.num_pages);
+    ctx->test_bad_page = 0;
+  }
   std::vector<int32_t> suf_off(n);
   for (int i = 0; i < n; ++i) {
     const Request& r = ctx->reqs[reqs[i]];
@@ -1580,6 +1586,9 @@ int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
       return TPA_OK;
     case TPA_OPT_TEST_PLAN_WAIT:
       ctx->test_plan_wait = value ? 1 : 0;
+      return TPA_OK;
+    case TPA_OPT_TEST_BAD_PAGE:
+      ctx->test_bad_page = value ? 1 : 0;
       return TPA_OK;
     case TPA_OPT_PREFILL_TILE_ROWS:
       if (value != 128 && value != 256) return fail(TPA_ERR_INVALID_ARG, "prefill tile rows %lld", (long long)value);

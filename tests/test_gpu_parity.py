@@ -259,6 +259,30 @@ def test_reload_rejects_unpinned_host_memory():
     assert s.ctx.query(B.Q_PREFIX_RESIDENT, 0) == 0
 
 
+@pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
+def test_out_of_pool_page_is_redirected_and_reported(mode):
+    # A plan whose first prefix page id lies outside the pool (test hook):
+    # every kernel bounds-checks page ids, so the read goes to page 0, the
+    # status word gets bit 4 and nothing faults; the next step is exact.
+    w = small_case(78, hq=8, hkv=2, d=128, prefix_len=[300, 40], req_agent=[0, 0, 1, 0],
+                   req_ctx=[10, 200, 33, 0], req_prefill=[0] * 4, req_decode=[1] * 4)
+    t, s = _session(w)
+    s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+    ids, q, kn, vn = s.decode_inputs()
+    lens = [s.ctx.query(B.Q_SUFFIX_LEN, r) for r in ids]
+    out, lse = s.new_outputs(len(ids))
+    s.ctx.set_option(B.OPT_TEST_BAD_PAGE, 1)
+    s.decode(ids, q, kn, vn, out, lse)
+    assert s.ctx.device_status() == 4
+    s.ctx.request_truncate(ids, lens)
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    ref = oracle.workload_decode(w, t)
+    o_ref, l_ref = stack_decode_ref(ref, range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "after an out-of-pool page id")
+
+
 def test_plan_wait_timeout_is_reported_and_context_recovers():
     # A decode whose kernel never sees its plan (test hook: the flag it waits
     # for is never written) gives up at the device wait limit; the host reads
