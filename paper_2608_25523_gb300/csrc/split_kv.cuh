@@ -18,9 +18,10 @@
 //    through ldmatrix.trans;
 //  * online softmax in base 2 with fp32 accumulators;
 //  * warps pull items from an atomic counter (items sorted longest first);
-//    a warp claims and resolves its next item, appends its token and loads
-//    its page ids while the current one streams, and keeps its ring full
-//    across the item boundary, so items cost no extra load latency.
+//    2 S pages before the current item ends a warp claims and resolves its
+//    next item, appends its token and loads its page ids, and keeps its ring
+//    full across the item boundary, so items cost no extra load latency,
+//    while the queue's tail stays unclaimed for warps that join it late.
 #pragma once
 #include "kernels.h"
 #include "ptx.cuh"
@@ -192,7 +193,12 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
   }
 
   while (idx < a.n_items) {
-    const uint32_t ticket = claim();  // the next item, claimed while this one streams
+    // The next item is claimed 2 S pages before this one ends (at once for a
+    // short item) and resolved right away, so its page loads follow this
+    // item's last pages without a gap; claiming later than that leaves the
+    // queue's tail to CTAs that join it late instead of piling it up behind
+    // busy warps.
+    const int claim_at = cur.npg > 2 * S ? cur.npg - 2 * S : 0;
     Work nxt{};
     int nxt_iss = 0;
     int idx_n = a.n_items;
@@ -292,9 +298,8 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
         }
       }
       __syncwarp();
-      if (pg == 0) {
-        // resolve the next item now: its loads overlap this item's stream
-        idx_n = __shfl_sync(0xffffffffu, static_cast<int>(ticket), 0);
+      if (pg == claim_at) {
+        idx_n = __shfl_sync(0xffffffffu, static_cast<int>(claim()), 0);
         if (idx_n < a.n_items) load_work(idx_n, nxt);
       }
       // refill the slot this page freed: this item's next page, else the next item's
