@@ -605,15 +605,34 @@ def bench_mixed(args, dev):
     side.synchronize()
     e1.synchronize()
     ms = e0.elapsed_time(e1) / k
+    # per-kernel device time (events around each launch, which also counts a
+    # launch's wait for free SMs, e.g. the reload scatter behind the prefill)
+    s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+    s.ctx.kernel_times(reset=True)
+    for _ in range(5):
+        step()
+    side.synchronize()
+    torch.cuda.synchronize(dev)
+    kt = s.ctx.kernel_times(reset=True)
     st = s.ctx.device_status()
     reload_bytes = sum(w.prefix_len[a] for a in w.reload_agents) * w.kv_bytes_per_token()
+    pf = prefill_flops(w, chunks)
+    _, _, dec_bytes = decode_bytes(w, dids)
     s.ctx.close()
+    per_step = {kk: {"us": round(1e3 * v[0] / 5, 1), "launches": v[1] // 5}
+                for kk, v in kt.items() if v[1]}
+    if "prefill_pair_tcgen05" in per_step:
+        per_step["prefill_pair_tcgen05"]["tflops"] = round(
+            pf / (per_step["prefill_pair_tcgen05"]["us"] * 1e-6) / 1e12, 1)
+    if "dense_tcgen05" in per_step:
+        per_step["dense_tcgen05"]["gbs"] = round(
+            dec_bytes / (per_step["dense_tcgen05"]["us"] * 1e-6) / 1e9, 1)
     return {"workload": "mixed: 16 agents prefixes U[1024,8192], 256 Zipf(1.1) decode requests "
                         "(suffixes U[256,1024]), 8 x 1024-token prefill chunks, permuted pool, "
                         "2 prefixes reloaded from pinned host on a side stream",
             "ms_per_step": round(ms, 4), "decode_tokens_per_s": round(len(dids) / (ms / 1e3), 1),
-            "prefill_flops": prefill_flops(w, chunks), "reload_bytes": reload_bytes,
-            "device_status": st}
+            "prefill_flops": pf, "decode_bytes": dec_bytes, "reload_bytes": reload_bytes,
+            "kernels_per_step": per_step, "device_status": st}
 
 
 def bench_movement(args, dev):

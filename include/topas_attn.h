@@ -94,7 +94,9 @@ typedef struct tpa_config {
 } tpa_config;
 
 /* Bytes of device workspace the context needs (plan ring, partial results,
- * status word).  Returns 0 for an invalid or unsupported configuration. */
+ * status word, and the prefix-movement staging area: K and V of a
+ * max_seq_len-token prefix).  Returns 0 for an invalid or unsupported
+ * configuration. */
 TPA_API size_t tpa_workspace_size(const tpa_config* cfg);
 
 /* Create a context over the caller's pools and workspace.  Builds the free
@@ -128,18 +130,23 @@ TPA_API int tpa_prefix_evict(tpa_ctx* ctx, int32_t agent);
 
 /* Prefix movement CPU -> GPU (Sec. IV-B, Eq. 7): take ceil(len/16) free
  * pages (in free-list order, so possibly scattered) and copy the pinned
- * host arrays bf16 [len][Hkv][d] `host_k`, `host_v` into them with a kernel
- * that reads host memory directly, on `side_stream`.  If `done_event` is
- * not NULL it is recorded after the copy.  Later calls that read this
- * prefix, on any stream, wait for the copy on the device.  Host memory must
- * be pinned (cudaHostAlloc / cudaHostRegister) and stay valid until the
- * copy completes.  Errors: INVALID_ARG (not pinned), STATE, NO_SPACE, CUDA. */
+ * host arrays bf16 [len][Hkv][d] `host_k`, `host_v` into them on
+ * `side_stream`: the copy engine moves them into the workspace's staging
+ * area, then a short kernel scatters them into the pages, so the transfer
+ * over the host link holds no SM.  Movement calls share the staging area
+ * and are ordered on the device.  If `done_event` is not NULL it is
+ * recorded after the copy.  Later calls that read this prefix, on any
+ * stream, wait for the copy on the device; a prefill call runs the chunks
+ * of other agents first.  Host memory must be pinned (cudaHostAlloc /
+ * cudaHostRegister) and stay valid until the copy completes.
+ * Errors: INVALID_ARG (not pinned), STATE, NO_SPACE, CUDA. */
 TPA_API int tpa_prefix_reload(tpa_ctx* ctx, int32_t agent, const void* host_k, const void* host_v,
                       void* side_stream, void* done_event);
 
 /* Prefix movement GPU -> CPU: copy a resident prefix into pinned host
- * arrays bf16 [len][Hkv][d] on `side_stream`, record `done_event` (if not
- * NULL), then evict it as tpa_prefix_evict does.  Errors as reload. */
+ * arrays bf16 [len][Hkv][d] on `side_stream` (a gather kernel into the
+ * staging area, then a copy-engine copy to the host), record `done_event`
+ * (if not NULL), then evict it as tpa_prefix_evict does.  Errors as reload. */
 TPA_API int tpa_prefix_offload(tpa_ctx* ctx, int32_t agent, void* host_k, void* host_v,
                        void* side_stream, void* done_event);
 

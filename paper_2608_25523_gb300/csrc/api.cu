@@ -147,6 +147,12 @@ struct tpa_ctx {
   uint32_t* status = nullptr;
   float* part_o = nullptr;
   float* part_lse = nullptr;
+  // staging area of the prefix movement: a whole prefix's K and V
+  // ([max_seq_len][Hkv][d] bf16 each); the host link transfer is a copy-engine
+  // copy into it, and the page scatter / gather an on-device kernel
+  uint8_t* stage_k = nullptr;
+  uint8_t* stage_v = nullptr;
+  uint64_t stage_seq = 0;  // the last movement call that used it
   int64_t part_slots = 0;
   size_t plan_cap = 0;               // bytes of a plan slot; its upload flag follows it
   Slot ring[kRingSlots];
@@ -244,6 +250,20 @@ void wait_for_seq(tpa_ctx* ctx, uint64_t seq, cudaStream_t s) {
     }
   }
   // not in the ring any more: its slot was recycled after a host-side wait
+}
+
+// Whether work on `s` would still have to wait for call `seq` (another
+// stream's call that has not completed).
+bool seq_pending(tpa_ctx* ctx, uint64_t seq, cudaStream_t s) {
+  if (seq == 0 || ctx->plan_only) return false;
+  for (auto& sl : ctx->ring) {
+    if (sl.seq != seq) continue;
+    if (sl.stream == s) return false;
+    if (cudaEventQuery(sl.done) == cudaErrorNotReady) return true;
+    (void)cudaGetLastError();
+    return false;
+  }
+  return false;
 }
 
 // Take `n` pages from the free list; returns the highest reuse tag.
@@ -430,6 +450,11 @@ extern "C" {
 
 const char* tpa_last_error(void) { return g_err.c_str(); }
 
+// One operand (K or V) of the longest prefix, [max_seq_len][Hkv][d] bf16.
+static size_t stage_bytes(const tpa_config* cfg) {
+  return static_cast<size_t>(cfg->max_seq_len) * cfg->num_kv_heads * cfg->head_dim * 2;
+}
+
 size_t tpa_workspace_size(const tpa_config* cfg) {
   if (!valid_shape(cfg) || cfg->max_tokens <= 0 || cfg->max_seq_len <= 0) return 0;
   const PlanLayout lay = layout_of(plan_capacity(cfg));
@@ -439,6 +464,7 @@ size_t tpa_workspace_size(const tpa_config* cfg) {
   total += kRingSlots * (align_up(lay.total, kAlign) + kAlign);  // plan ring (+ upload flags)
   total += align_up(slots * cfg->head_dim * sizeof(float), kAlign);
   total += align_up(slots * sizeof(float), kAlign);
+  total += 2 * align_up(stage_bytes(cfg), kAlign);           // prefix movement staging
   return total;
 }
 
@@ -579,6 +605,10 @@ int tpa_create(const tpa_config* cfg, tpa_ctx** out) {
   ctx->part_o = reinterpret_cast<float*>(ws + off);
   off += align_up(ctx->part_slots * ctx->d * sizeof(float), kAlign);
   ctx->part_lse = reinterpret_cast<float*>(ws + off);
+  off += align_up(ctx->part_slots * sizeof(float), kAlign);
+  ctx->stage_k = ws + off;
+  off += align_up(stage_bytes(cfg), kAlign);
+  ctx->stage_v = ws + off;
 
   for (auto& s : ctx->ring) {
     if ((e = cudaHostAlloc(reinterpret_cast<void**>(&s.host), ctx->plan_cap + kAlign,
@@ -648,9 +678,18 @@ int tpa_prefix_register(tpa_ctx* ctx, int32_t agent, int32_t len) {
   return TPA_OK;
 }
 
+// Copy `len` tokens between a contiguous [len][Hkv][d] pair of arrays and a
+// page run.  `staged`: the contiguous side is host memory, moved by the copy
+// engine through the workspace's staging area while the page scatter (to
+// pages) or gather (from pages) is a short on-device kernel, so the link
+// transfer holds no SM while compute runs beside it; otherwise the kernel
+// reads or writes the contiguous side itself.
 static int page_copy_call(tpa_ctx* ctx, const std::vector<int32_t>& pages, int len, int to_pages,
                           const void* k_in, const void* v_in, void* k_out, void* v_out,
-                          cudaStream_t s, bool chain, uint64_t wait_seq, Slot** used) {
+                          cudaStream_t s, bool chain, uint64_t wait_seq, Slot** used,
+                          bool staged = false) {
+  const size_t bytes = static_cast<size_t>(len) * ctx->hkv * ctx->d * 2;
+  if (staged && len > ctx->cfg.max_seq_len) return fail(TPA_ERR_CAPACITY, "%d tokens > max_seq_len", len);
   Slot* sl = acquire_slot(ctx);
   ++ctx->seq;
   PlanSizes sz;
@@ -662,13 +701,29 @@ static int page_copy_call(tpa_ctx* ctx, const std::vector<int32_t>& pages, int l
   std::memcpy(w.pages, pages.data(), pages.size() * 4);
   if (chain) chain_begin(ctx, s);
   wait_for_seq(ctx, wait_seq, s);
+  if (staged) wait_for_seq(ctx, ctx->stage_seq, s);  // the staging area's previous user
   int rc = upload(ctx, sl, lay.total, s);
   if (rc) return rc;
   if (!ctx->plan_only) {
-    KernelTimer kt(ctx, K_COPY, s);
-    CUDA_TRY(launch_page_copy(dev_ptr<int32_t>(sl, lay.off_pages), len, to_pages, k_in, v_in, k_out,
-                              v_out, ctx->pool, ctx->status, s));
+    const bool in = staged && to_pages && len > 0, out = staged && !to_pages && len > 0;
+    if (in) {
+      CUDA_TRY(cudaMemcpyAsync(ctx->stage_k, k_in, bytes, cudaMemcpyDefault, s));
+      CUDA_TRY(cudaMemcpyAsync(ctx->stage_v, v_in, bytes, cudaMemcpyDefault, s));
+      k_in = ctx->stage_k;
+      v_in = ctx->stage_v;
+    }
+    {
+      KernelTimer kt(ctx, K_COPY, s);
+      CUDA_TRY(launch_page_copy(dev_ptr<int32_t>(sl, lay.off_pages), len, to_pages, k_in, v_in,
+                                out ? ctx->stage_k : k_out, out ? ctx->stage_v : v_out, ctx->pool,
+                                ctx->status, s));
+    }
+    if (out) {
+      CUDA_TRY(cudaMemcpyAsync(k_out, ctx->stage_k, bytes, cudaMemcpyDefault, s));
+      CUDA_TRY(cudaMemcpyAsync(v_out, ctx->stage_v, bytes, cudaMemcpyDefault, s));
+    }
   }
+  if (staged) ctx->stage_seq = ctx->seq;
   ctx->last_launches = 1;
   if (used) *used = sl;
   return finish_call(ctx, sl, s, chain);
@@ -751,8 +806,8 @@ int tpa_prefix_reload(tpa_ctx* ctx, int32_t agent, const void* host_k, const voi
   std::vector<int32_t> pages;
   const uint64_t tag = take_pages(ctx, need, pages);
   cudaStream_t s = static_cast<cudaStream_t>(side_stream);
-  const int rc = page_copy_call(ctx, pages, a.len, 1, kd, vd, nullptr, nullptr, s, false,
-                                std::max(tag, a.last_use), nullptr);
+  const int rc = page_copy_call(ctx, pages, a.len, 1, host_k, host_v, nullptr, nullptr, s, false,
+                                std::max(tag, a.last_use), nullptr, true);
   if (rc) {
     // give the pages back untouched (nothing was queued that writes them)
     for (auto it = pages.rbegin(); it != pages.rend(); ++it) ctx->free_pages[--ctx->free_head] = *it;
@@ -783,9 +838,8 @@ int tpa_prefix_offload(tpa_ctx* ctx, int32_t agent, void* host_k, void* host_v, 
   cudaStream_t s = static_cast<cudaStream_t>(side_stream);
   // the pages' last writer/readers must finish before the copy reads them
   wait_for_seq(ctx, ctx->chain_seq, s);
-  const int rc = page_copy_call(ctx, a.pages, a.len, 0, nullptr, nullptr, const_cast<void*>(kd),
-                                const_cast<void*>(vd), s, false, std::max(a.ready_seq, a.last_use),
-                                nullptr);
+  const int rc = page_copy_call(ctx, a.pages, a.len, 0, nullptr, nullptr, host_k, host_v, s, false,
+                                std::max(a.ready_seq, a.last_use), nullptr, true);
   if (rc) return rc;
   a.last_use = ctx->seq;
   give_pages(ctx, a.pages, ctx->seq);
@@ -1360,8 +1414,22 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   const bool pairs = ctx->prefill_rows == 2 * kTileRows;
   const int tpt = (pairs ? 2 * kTileRows : kTileRows) / G;  // tokens per work item
 
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
   std::vector<int32_t> offset(n);
   for (int i = 0; i < n; ++i) offset[i] = ctx->reqs[reqs[i]].len;
+  // Chunks of an agent whose prefix reload (on another stream) is still in
+  // flight run in a second launch after the stream waits for that reload;
+  // the other chunks' items run meanwhile.  Only the requests that need an
+  // incoming prefix wait for its movement (Sec. IV-B, Eq. 7).
+  std::vector<uint8_t> late(n, 0);
+  {
+    bool any_early = false, any_late = false;
+    for (int i = 0; i < n; ++i) {
+      late[i] = seq_pending(ctx, ctx->agents[ctx->reqs[reqs[i]].agent].ready_seq, s) ? 1 : 0;
+      (late[i] ? any_late : any_early) = true;
+    }
+    if (!any_early || !any_late) std::fill(late.begin(), late.end(), 0);
+  }
 
   std::vector<int32_t> agents_seen;
   PlanSizes sz;
@@ -1404,6 +1472,29 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
       }
     }
   }
+  // Items go straight to their place, the early chunks' items first, each
+  // group in longest-first order (a stable counting sort on the key-tile
+  // count): first count the items of each length, then write them.
+  auto tiles_of = [&](int i, int t1) {
+    const int64_t lp = ctx->agents[ctx->reqs[reqs[i]].agent].len;
+    return static_cast<int32_t>(cdiv(lp, kTileKeys) + cdiv(offset[i] + t1, kTileKeys));
+  };
+  int32_t max_tiles = 0;  // a request's last tile has the most keys
+  for (int i = 0; i < n; ++i) max_tiles = std::max(max_tiles, tiles_of(i, chunk_len[i]));
+  const size_t n_len = static_cast<size_t>(max_tiles) + 1;
+  std::vector<int32_t> at(2 * n_len, 0);  // [group][key tiles]
+  for (int i = 0; i < n; ++i)
+    for (int t0 = 0; t0 < chunk_len[i]; t0 += tpt)
+      at[late[i] * n_len + tiles_of(i, std::min(chunk_len[i], t0 + tpt))] += hkv;
+  int32_t n_early = 0;
+  for (int g = 0, acc = 0; g < 2; ++g) {  // exclusive prefix, longest first
+    for (size_t k = n_len; k-- > 0;) {
+      const int32_t c = at[g * n_len + k];
+      at[g * n_len + k] = acc;
+      acc += c;
+    }
+    if (g == 0) n_early = acc;
+  }
   int32_t nt = 0, nd = 0;
   int64_t row0 = 0;
   for (int i = 0; i < n; ++i) {
@@ -1418,37 +1509,37 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
       const int32_t tok_base = nt;
       for (int t = t0; t < t1; ++t)
         w.dtok[nt++] = DenseTok{static_cast<int32_t>(row0 + t), offset[i] + t, 0, 0};
+      DenseItem it{};
+      it.tok_base = tok_base;
+      it.n_tok = t1 - t0;
+      it.out_mode = 1;
+      it.seg_pages[0] = agent_off[r.agent];
+      it.seg_k0[0] = 0;
+      it.seg_k1[0] = static_cast<int32_t>(lp);
+      it.seg_pages[1] = suf;
+      it.seg_k0[1] = 0;
+      it.seg_k1[1] = offset[i] + t1;  // keys up to the tile's last position
+      it.seg_causal[1] = 1;
+      it.n_tiles = tiles_of(i, t1);
+      int32_t& pos = at[late[i] * n_len + it.n_tiles];
+      DenseItem* dst = w.dense + pos;
+      pos += hkv;
       for (int h = 0; h < hkv; ++h) {
-        DenseItem it{};
-        it.tok_base = tok_base;
-        it.n_tok = t1 - t0;
         it.kv_head = h;
-        it.out_mode = 1;
-        it.seg_pages[0] = agent_off[r.agent];
-        it.seg_k0[0] = 0;
-        it.seg_k1[0] = static_cast<int32_t>(lp);
-        it.seg_pages[1] = suf;
-        it.seg_k0[1] = 0;
-        it.seg_k1[1] = offset[i] + t1;  // keys up to the tile's last position
-        it.seg_causal[1] = 1;
-        it.n_tiles = static_cast<int32_t>(cdiv(lp, kTileKeys) + cdiv(it.seg_k1[1], kTileKeys));
-        w.dense[nd++] = it;
+        dst[h] = it;
       }
+      nd += hkv;
     }
     row0 += c;
   }
-  std::stable_sort(w.dense, w.dense + nd,
-                   [](const DenseItem& a, const DenseItem& b) { return a.n_tiles > b.n_tiles; });
   PlanHeader* hd = w.hdr;
   hd->n_pages = np;
   hd->n_append = static_cast<int32_t>(total);
   hd->n_dense_tok = nt;
   hd->n_dense = nd;
 
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   chain_begin(ctx, s);
   wait_for_seq(ctx, tag, s);
-  for (int32_t a : agents_seen) wait_for_seq(ctx, ctx->agents[a].ready_seq, s);
   if ((rc = upload(ctx, sl, lay.total, s))) return rc;
   if (!ctx->plan_only) {
     {
@@ -1456,13 +1547,22 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
       CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
                              v_new, ctx->pool, ctx->status, s));
     }
-    DenseParams dp = dense_params(ctx, sl, lay, nd, q, out, lse);
-    dp.n_dense_ctas = std::min(nd, ctx->num_sms);
-    KernelTimer kt(ctx, pairs ? K_PREFILL_PAIR : K_DENSE, s);
-    if (pairs)
-      CUDA_TRY(launch_prefill_pair(dp, dp.n_dense_ctas, ctx->d, G, s));
-    else
-      CUDA_TRY(launch_dense(dp, 0, ctx->d, G, false, s));
+    // items [0, n_early) after the reloads of their agents (if any is
+    // still pending, no chunk is late), then the late ones after theirs
+    for (int g = 0; g < 2; ++g) {
+      const int32_t i0 = g == 0 ? 0 : n_early, i1 = g == 0 ? n_early : nd;
+      for (int i = 0; i < n; ++i)
+        if (late[i] == g) wait_for_seq(ctx, ctx->agents[ctx->reqs[reqs[i]].agent].ready_seq, s);
+      if (i1 == i0) continue;
+      DenseParams dp = dense_params(ctx, sl, lay, i1 - i0, q, out, lse);
+      dp.items += i0;
+      dp.n_dense_ctas = std::min(i1 - i0, ctx->num_sms);
+      KernelTimer kt(ctx, pairs ? K_PREFILL_PAIR : K_DENSE, s);
+      if (pairs)
+        CUDA_TRY(launch_prefill_pair(dp, dp.n_dense_ctas, ctx->d, G, s));
+      else
+        CUDA_TRY(launch_dense(dp, 0, ctx->d, G, false, s));
+    }
   }
   for (int i = 0; i < n; ++i) {
     Request& r = ctx->reqs[reqs[i]];

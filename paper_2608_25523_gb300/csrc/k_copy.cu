@@ -4,12 +4,13 @@
 //    appends) go to (page, slot) positions chosen by the host planner.
 //    Suffixes start on a fresh page, so shared prefix pages are never
 //    written by a request (the prefix is paid once per agent, Eq. 2).
-//  * page copy: a contiguous [len][Hkv][d] prefix <-> its page run.  This is
-//    the prefix movement between CPU and GPU memory (Sec. IV-B, Eq. 7):
-//    with a mapped pinned-host source it is the reload scatter, with a
-//    pinned-host destination the offload gather.  Host memory is read or
-//    written directly by the kernel over the CPU-GPU link, so a fragmented
-//    (permuted) page run costs no extra copies.
+//  * page copy: a contiguous [len][Hkv][d] prefix <-> its page run, in
+//    either direction.  The prefix movement between CPU and GPU memory
+//    (Sec. IV-B, Eq. 7) uses it on the device side of a copy-engine
+//    transfer: the reload scatters a staged prefix into free, possibly
+//    fragmented pages, the offload gathers the pages into the staging area.
+//    Prefix writes from device (or mapped pinned host) arrays use it
+//    directly.
 // Every copy moves 16-byte units; consecutive threads take consecutive
 // units of one token row, so both sides are coalesced.
 #include "kernels.h"
@@ -20,27 +21,47 @@ namespace {
 
 constexpr int kCopyThreads = 256;
 
+constexpr int kAppendUnroll = 4;
+
+// Unit x of the call (32-bit: the host checks the count) is 16-byte unit
+// x % upr of row x / upr, where a row is one token's K (or V) across the kv
+// heads; each thread loads kAppendUnroll units of K and of V before it
+// stores any, so enough bytes are in flight to stream at HBM rate.
+template <int CPR>
 __global__ void __launch_bounds__(kCopyThreads)
     append_kernel(const AppendRow* __restrict__ rows, int n_rows, const uint4* __restrict__ k_src,
                   const uint4* __restrict__ v_src, uint4* __restrict__ k_pool,
-                  uint4* __restrict__ v_pool, int64_t num_pages, int hkv, int cpr,
-                  uint32_t* status) {
-  const int64_t total = static_cast<int64_t>(n_rows) * hkv * cpr;
-  for (int64_t u = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; u < total;
-       u += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int c = static_cast<int>(u % cpr);
-    const int64_t t = u / cpr;
-    const int h = static_cast<int>(t % hkv);
-    const int row = static_cast<int>(t / hkv);
-    const AppendRow r = rows[row];
-    if (r.page < 0 || r.page >= num_pages || r.slot < 0 || r.slot >= kPage) {
-      atomicOr(status, kStatusBadPage);
-      continue;
+                  uint4* __restrict__ v_pool, int64_t num_pages, int hkv, uint32_t* status) {
+  const int upr = hkv * CPR;
+  const int total = n_rows * upr;
+  const int stride = gridDim.x * blockDim.x;
+  for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < total; u += kAppendUnroll * stride) {
+    uint4 kx[kAppendUnroll], vx[kAppendUnroll];
+    int64_t dst[kAppendUnroll];
+#pragma unroll
+    for (int i = 0; i < kAppendUnroll; ++i) {
+      dst[i] = -1;
+      const int x = u + i * stride;
+      if (x >= total) continue;
+      const int row = x / upr;
+      const int rem = x - row * upr;
+      const AppendRow r = rows[row];
+      if (r.page < 0 || r.page >= num_pages || r.slot < 0 || r.slot >= kPage) {
+        atomicOr(status, kStatusBadPage);
+        continue;
+      }
+      const int h = rem / CPR, c = rem % CPR;
+      dst[i] = ((static_cast<int64_t>(r.page) * hkv + h) * kPage + r.slot) * CPR + c;
+      const int64_t src = static_cast<int64_t>(r.src) * upr + rem;
+      kx[i] = k_src[src];
+      vx[i] = v_src[src];
     }
-    const int64_t src = (static_cast<int64_t>(r.src) * hkv + h) * cpr + c;
-    const int64_t dst = ((static_cast<int64_t>(r.page) * hkv + h) * kPage + r.slot) * cpr + c;
-    k_pool[dst] = k_src[src];
-    v_pool[dst] = v_src[src];
+#pragma unroll
+    for (int i = 0; i < kAppendUnroll; ++i) {
+      if (dst[i] < 0) continue;
+      k_pool[dst[i]] = kx[i];
+      v_pool[dst[i]] = vx[i];
+    }
   }
 }
 
@@ -89,10 +110,18 @@ cudaError_t launch_append(const AppendRow* rows, int n_rows, const void* k_src,
   if (n_rows <= 0) return cudaSuccess;
   const int cpr = pool.d / 8;
   const int64_t units = static_cast<int64_t>(n_rows) * pool.hkv * cpr;
-  append_kernel<<<copy_grid(units), kCopyThreads, 0, stream>>>(
-      rows, n_rows, static_cast<const uint4*>(k_src), static_cast<const uint4*>(v_src),
-      static_cast<uint4*>(pool.k), static_cast<uint4*>(pool.v), pool.num_pages, pool.hkv, cpr,
-      status);
+  if (units > INT32_MAX || (cpr != 8 && cpr != 16)) return cudaErrorInvalidValue;
+  const int grid = copy_grid((units + kAppendUnroll - 1) / kAppendUnroll);
+  auto* const ks = static_cast<const uint4*>(k_src);
+  auto* const vs = static_cast<const uint4*>(v_src);
+  auto* const kp = static_cast<uint4*>(pool.k);
+  auto* const vp = static_cast<uint4*>(pool.v);
+  if (cpr == 16)
+    append_kernel<16><<<grid, kCopyThreads, 0, stream>>>(rows, n_rows, ks, vs, kp, vp,
+                                                         pool.num_pages, pool.hkv, status);
+  else
+    append_kernel<8><<<grid, kCopyThreads, 0, stream>>>(rows, n_rows, ks, vs, kp, vp,
+                                                        pool.num_pages, pool.hkv, status);
   return cudaGetLastError();
 }
 

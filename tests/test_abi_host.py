@@ -220,6 +220,22 @@ def test_prefill_plan_decomposition(lib):
         ctx.set_option(B.OPT_PREFILL_TILE_ROWS, 64)
 
 
+def test_prefill_plan_with_prefix_and_suffix_at_max_seq_len(lib):
+    """An item's key tiles (prefix + causal suffix) can reach twice
+    max_seq_len / 128; the planner's longest-first ordering must size for
+    that."""
+    hkv, G = 2, 4
+    ctx = plan_ctx(num_pages=300, hq=8, hkv=hkv, agents=2, reqs=3, tokens=2048, seq=1024)
+    ctx.prefix_register(0, 1024)
+    ctx.prefix_register(1, 1000)
+    for r, a in enumerate((0, 1, 0)):
+        ctx.request_open(r, a)
+    for c in (1000, 24):
+        ctx.prefill_chunk([0, 1, 2], [c, c, 1], 1, 1, 1, 1, 1)
+        assert ctx.query(B.Q_LAST_DENSE_ITEMS) == hkv * (2 * math.ceil(c / (256 // G)) + 1)
+    assert [ctx.query(B.Q_SUFFIX_LEN, r) for r in range(3)] == [1024, 1024, 2]
+
+
 def test_permuted_pool_is_a_permutation(lib):
     ctx = plan_ctx(num_pages=50, seed=12345)
     firsts = []

@@ -247,6 +247,44 @@ def test_offload_reload_bit_exact_on_side_stream():
     assert torch.equal(_bits(k), _bits(pk)) and torch.equal(_bits(v), _bits(pv))
 
 
+@pytest.mark.parametrize("rows", [256, 128], ids=["pairs", "single"])
+def test_prefill_runs_ready_chunks_before_a_pending_reload(rows):
+    """A prefill call whose chunks include an agent with a reload still in
+    flight on a side stream: the other agents' items run in a first launch,
+    the reloading agent's in a second one after the stream waits for the
+    reload.  Every chunk must still match the oracle."""
+    w = small_case(29, hq=8, hkv=2, d=128, prefix_len=[333, 200, 48],
+                   req_agent=[0, 1, 2, 0, 1], req_ctx=[0] * 5, req_prefill=[100, 70, 64, 40, 90],
+                   req_decode=[0] * 5, chunk=128, permute=True)
+    t, s = _session(w)
+    s.ctx.set_option(B.OPT_PREFILL_TILE_ROWS, rows)
+    L = w.prefix_len[0]
+    hk = torch.empty(L, 2, 128, dtype=torch.bfloat16, pin_memory=True)
+    hv = torch.empty_like(hk, pin_memory=True)
+    side = torch.cuda.Stream()
+    ev = torch.cuda.Event()
+    s.ctx.prefix_offload(0, hk, hv, side, ev)
+    ev.synchronize()
+    chunks, ids, lens, q, k, v = s.prefill_inputs(0)
+    out, lse = s.new_outputs(sum(lens))
+    torch.cuda.synchronize()
+    s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+    s.ctx.kernel_times(reset=True)
+    with torch.cuda.stream(side):
+        torch.cuda._sleep(20_000_000)   # keeps the reload behind it in flight (bounded spin)
+    s.ctx.prefix_reload(0, hk, hv, side, None)
+    s.prefill(ids, lens, q, k, v, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    kt = s.ctx.kernel_times(reset=True)
+    assert kt["prefill_pair_tcgen05" if rows == 256 else "dense_tcgen05"][1] == 2
+    row = 0
+    for r, off, c in chunks:
+        o_ref, l_ref = oracle.workload_prefill_chunk(w, t, r, off, c)
+        compare(out[row:row + c], lse[row:row + c], o_ref, l_ref, f"r{r} off{off}")
+        row += c
+
+
 def test_reload_rejects_unpinned_host_memory():
     w = small_case(25, hq=8, hkv=2, d=64, prefix_len=[40], req_agent=[0], req_ctx=[1],
                    req_prefill=[0], req_decode=[1])
