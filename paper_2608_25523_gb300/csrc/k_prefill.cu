@@ -163,38 +163,53 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
         if (ok && !mbar_wait(&bars[b], parity, ab)) ok = false;
         return ok;
       };
-      // S_X = Q_X K_g^T; the last QK of tile g (X = 1) releases K stage g % 3
-      auto issue_qk = [&](int x, int g) {
-        const int ks = g % C::kStagesK;
+      // The issuing thread stays lean: the tensor pipe accepts a new MMA only
+      // as an earlier one retires, so any work between MMAs (descriptor
+      // arithmetic, a barrier wait inside a group) leaves it idle.  The
+      // descriptors of kk = 0 are built once; a kk step or a ring stage adds
+      // its byte offset / 16 to the start-address field (bits 0-13, no carry:
+      // shared addresses stay below 256 KB).  K and V tiles are consumed in
+      // order through running stage / phase counters.
+      const uint64_t dq0 = umma_sdesc(qbase, 16, 1024);
+      const uint64_t dk0 = umma_sdesc(kbase, 16, T::kGroup);
+      const uint64_t dv0 = umma_sdesc(vbase, 1024, T::kGroup);
+      int ks = 0, vs = 0;          // ring stage of the next K tile / the current V tile
+      uint32_t kph = 0, vph = 0;   // their full-barrier phases
+      // S_X = Q_X K^T with K from stage ks; the tile's second QK (X = 1)
+      // releases the stage
+      auto issue_qk = [&](int x) {
         tc_fence_after();
-        const uint32_t kb = kbase + ks * T::kBytes;
-        const uint32_t qb = qbase + x * C::kQBytes;
+        const uint64_t a0 = dq0 + static_cast<uint64_t>((x * C::kQBytes) >> 4);
+        const uint64_t b0 = dk0 + static_cast<uint64_t>((ks * T::kBytes) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t a = umma_sdesc(qb + (kk >> 2) * T::kChunk + (kk & 3) * 32, 16, 1024);
-          const uint64_t b = umma_sdesc(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, T::kGroup);
-          umma_bf16_ss(tmem + x * 128, a, b, idesc_qk, kk > 0 ? 1u : 0u);
-        }
+        for (int kk = 0; kk < D / 16; ++kk)
+          umma_bf16_ss(tmem + x * 128, a0 + (((kk >> 2) * T::kChunk + (kk & 3) * 32) >> 4),
+                       b0 + (((kk >> 2) * 1024 + (kk & 3) * 32) >> 4), idesc_qk, kk > 0 ? 1u : 0u);
         umma_commit(&bars[C::B_SFULL + x]);
-        if (x == 1) umma_commit(&bars[C::B_KEMPTY + ks]);
+        if (x == 1) {
+          umma_commit(&bars[C::B_KEMPTY + ks]);
+          if (++ks == C::kStagesK) { ks = 0; kph ^= 1u; }
+        }
       };
-      // O_X (+)= P_X V_g with P_X from the first 64 columns of S_X; the last
-      // PV of tile g (X = 1) releases V stage g % S_V
-      auto issue_pv = [&](int x, int g, bool first) {
-        const int vs = g % C::kStagesV;
+      // O_X (+)= P_X V with P_X from the first 64 columns of S_X and V from
+      // stage vs; the tile's second PV (X = 1) releases the stage
+      auto issue_pv = [&](int x, bool first) {
         tc_fence_after();
-        const uint32_t vb = vbase + vs * T::kBytes;
+        const uint64_t b0 = dv0 + static_cast<uint64_t>((vs * T::kBytes) >> 4);
         const uint32_t pcol = tmem + x * 128;
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t b = umma_sdesc(vb + kk * T::kPageBytes, 1024, T::kGroup);
-          umma_bf16_ts(tmem + C::kColO + x * D, pcol + kk * 8, b, idesc_pv, (!first || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < 8; ++kk)
+          umma_bf16_ts(tmem + C::kColO + x * D, pcol + kk * 8, b0 + ((kk * T::kPageBytes) >> 4),
+                       idesc_pv, (!first || kk > 0) ? 1u : 0u);
         umma_commit(&bars[C::B_PVDONE + x]);
-        if (x == 1) umma_commit(&bars[C::B_VEMPTY + vs]);
+        if (x == 1) {
+          umma_commit(&bars[C::B_VEMPTY + vs]);
+          if (++vs == C::kStagesV) { vs = 0; vph ^= 1u; }
+        }
       };
       // The CTA's tiles in order, g counting across items; the first tile of
-      // item k waits for both Q tiles of the item (phase k).
+      // item k waits for both Q tiles of the item (phase k).  All waits of a
+      // group come before its MMAs.
       int g = 0;
       for (int k = 0; ok; ++k) {
         const int idx = item_of(k, n_ctas);
@@ -208,23 +223,19 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
           if (j == 0) {
             // this item's S_A(0), S_B(0); the previous item's last PVs were
             // issued before them
-            if (!wait(C::B_KFULL + g % C::kStagesK, (g / C::kStagesK) & 1)) break;
-            if (!wait(C::B_QFULL + 0, k & 1)) break;
-            issue_qk(0, g);
+            if (!wait(C::B_KFULL + ks, kph) || !wait(C::B_QFULL + 0, k & 1)) break;
+            issue_qk(0);
             if (!wait(C::B_QFULL + 1, k & 1)) break;
-            issue_qk(1, g);
+            issue_qk(1);
           }
           const bool more = j + 1 < ntiles;
-          if (!wait(C::B_PFULL + 0, g & 1)) break;
-          if (!wait(C::B_VFULL + g % C::kStagesV, (g / C::kStagesV) & 1)) break;
-          issue_pv(0, g, j == 0);
-          if (more) {
-            if (!wait(C::B_KFULL + (g + 1) % C::kStagesK, ((g + 1) / C::kStagesK) & 1)) break;
-            issue_qk(0, g + 1);
-          }
+          if (!wait(C::B_PFULL + 0, g & 1) || !wait(C::B_VFULL + vs, vph)) break;
+          if (more && !wait(C::B_KFULL + ks, kph)) break;
+          issue_pv(0, j == 0);
+          if (more) issue_qk(0);
           if (!wait(C::B_PFULL + 1, g & 1)) break;
-          issue_pv(1, g, j == 0);
-          if (more) issue_qk(1, g + 1);
+          issue_pv(1, j == 0);
+          if (more) issue_qk(1);
         }
       }
       if (!ok) {
