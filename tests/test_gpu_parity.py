@@ -247,6 +247,44 @@ def test_offload_reload_bit_exact_on_side_stream():
     assert torch.equal(_bits(k), _bits(pk)) and torch.equal(_bits(v), _bits(pv))
 
 
+def test_concurrent_reloads_on_two_streams_share_the_staging_area():
+    """Two prefixes reloaded at once on two side streams go through the one
+    staging area of the workspace; the second waits for the first on the
+    device.  Both land bit-exact and a decode over them matches the oracle."""
+    w = small_case(31, hq=8, hkv=2, d=128, prefix_len=[500, 333, 17], req_agent=[0, 1, 2, 0, 1],
+                   req_ctx=[20, 5, 77, 3, 40], req_prefill=[0] * 5, req_decode=[1] * 5, permute=True)
+    t, s = _session(w)
+    hosts = {}
+    side = [torch.cuda.Stream(), torch.cuda.Stream()]
+    for a in (0, 1):
+        L = w.prefix_len[a]
+        hk = torch.empty(L, 2, 128, dtype=torch.bfloat16, pin_memory=True)
+        hv = torch.empty_like(hk, pin_memory=True)
+        ev = torch.cuda.Event()
+        s.ctx.prefix_offload(a, hk, hv, side[a], ev)
+        ev.synchronize()
+        hosts[a] = (hk, hv)
+    with torch.cuda.stream(side[0]):
+        torch.cuda._sleep(5_000_000)   # the first reload is still in flight when the second is issued
+    for a in (0, 1):
+        s.ctx.prefix_reload(a, hosts[a][0], hosts[a][1], side[a], None)
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "after two reloads")
+    for a in (0, 1):
+        L = w.prefix_len[a]
+        k = torch.empty(L, 2, 128, dtype=torch.bfloat16, device="cuda")
+        v = torch.empty_like(k)
+        s.ctx.gather(a, False, k, v)
+        pk, pv = s.t.prefix(a, w)
+        torch.cuda.synchronize()
+        assert torch.equal(_bits(k), _bits(pk)) and torch.equal(_bits(v), _bits(pv)), a
+
+
 @pytest.mark.parametrize("rows", [256, 128], ids=["pairs", "single"])
 def test_prefill_runs_ready_chunks_before_a_pending_reload(rows):
     """A prefill call whose chunks include an agent with a reload still in
