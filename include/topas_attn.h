@@ -196,8 +196,14 @@ TPA_API int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, cons
 /* One decode step for `n` distinct open requests with resident prefixes:
  * append each request's new token K/V, then attend each query to its
  * prefix, its suffix and the new token.
- *   q      device bf16 [n][Hq][d];   k_new, v_new device bf16 [n][Hkv][d]
- *   out    device bf16 [n][Hq][d];   lse device fp32 [n][Hq]
+ *   q      bf16 [n][Hq][d];   k_new, v_new bf16 [n][Hkv][d]
+ *   out    bf16 [n][Hq][d];   lse fp32 [n][Hq]
+ * These five arrays are device memory, or pinned host memory from
+ * cudaHostAlloc (mapped: its host address is its device address).  With
+ * host memory the kernels read the step's inputs and write its outputs
+ * over the CPU-GPU link themselves, with no staging copy; the results are
+ * bit-identical to the device-memory call.  The caller keeps host arrays
+ * valid and unread until the stream passes the call.
  * Errors: INVALID_ARG, STATE, NOT_RESIDENT, NO_SPACE, CAPACITY, CUDA. */
 TPA_API int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q,
                const void* k_new, const void* v_new, void* out, float* lse, void* stream);

@@ -247,6 +247,38 @@ def test_offload_reload_bit_exact_on_side_stream():
     assert torch.equal(_bits(k), _bits(pk)) and torch.equal(_bits(v), _bits(pv))
 
 
+def test_decode_with_pinned_host_io_is_bit_identical():
+    """q, k_new, v_new, out, lse in pinned host memory: the kernels read and
+    write them over the host link, and the outputs and the appended pages
+    equal those of the same step with device buffers bit for bit."""
+    w = small_case(37, hq=8, hkv=2, d=128, prefix_len=[300, 17], req_agent=[0, 1, 0, 1, 0],
+                   req_ctx=[10, 200, 0, 33, 97], req_prefill=[0] * 5, req_decode=[1] * 5,
+                   permute=True)
+    t, s = _session(w)
+    ids, q, kn, vn = s.decode_inputs()
+    lens = [w.req_ctx[r] for r in ids]
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    k_dev = torch.empty(w.req_ctx[ids[0]] + 1, 2, 128, dtype=torch.bfloat16, device="cuda")
+    v_dev = torch.empty_like(k_dev)
+    s.ctx.gather(ids[0], True, k_dev, v_dev)
+    s.ctx.request_truncate(ids, lens)
+    pin = lambda x: x.cpu().pin_memory()
+    hq, hk, hv = pin(q), pin(kn), pin(vn)
+    ho = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+    hl = torch.empty(lse.shape, dtype=lse.dtype, pin_memory=True)
+    s.decode(ids, hq, hk, hv, ho, hl)
+    k2 = torch.empty_like(k_dev)
+    v2 = torch.empty_like(v_dev)
+    s.ctx.gather(ids[0], True, k2, v2)
+    torch.cuda.synchronize()
+    _check_status(s)
+    assert torch.equal(_bits(ho), _bits(out.cpu())) and torch.equal(hl, lse.cpu())
+    assert torch.equal(_bits(k2), _bits(k_dev)) and torch.equal(_bits(v2), _bits(v_dev))
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(ho, hl, o_ref, l_ref, "pinned host io")
+
+
 def test_concurrent_reloads_on_two_streams_share_the_staging_area():
     """Two prefixes reloaded at once on two side streams go through the one
     staging area of the workspace; the second waits for the first on the
