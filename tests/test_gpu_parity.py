@@ -317,15 +317,19 @@ def test_concurrent_reloads_on_two_streams_share_the_staging_area():
         assert torch.equal(_bits(k), _bits(pk)) and torch.equal(_bits(v), _bits(pv)), a
 
 
+@pytest.mark.parametrize("only_reloading", [False, True], ids=["mixed_agents", "only_reloading"])
 @pytest.mark.parametrize("rows", [256, 128], ids=["pairs", "single"])
-def test_prefill_runs_ready_chunks_before_a_pending_reload(rows):
+def test_prefill_runs_ready_chunks_before_a_pending_reload(rows, only_reloading):
     """A prefill call whose chunks include an agent with a reload still in
     flight on a side stream: the other agents' items run in a first launch,
     the reloading agent's in a second one after the stream waits for the
-    reload.  Every chunk must still match the oracle."""
+    reload.  When every chunk belongs to the reloading agent there is one
+    launch, after the wait.  Every chunk must still match the oracle."""
+    agents = [0, 0, 0] if only_reloading else [0, 1, 2, 0, 1]
     w = small_case(29, hq=8, hkv=2, d=128, prefix_len=[333, 200, 48],
-                   req_agent=[0, 1, 2, 0, 1], req_ctx=[0] * 5, req_prefill=[100, 70, 64, 40, 90],
-                   req_decode=[0] * 5, chunk=128, permute=True)
+                   req_agent=agents, req_ctx=[0] * len(agents),
+                   req_prefill=[100, 70, 64, 40, 90][:len(agents)],
+                   req_decode=[0] * len(agents), chunk=128, permute=True)
     t, s = _session(w)
     s.ctx.set_option(B.OPT_PREFILL_TILE_ROWS, rows)
     L = w.prefix_len[0]
@@ -347,7 +351,7 @@ def test_prefill_runs_ready_chunks_before_a_pending_reload(rows):
     torch.cuda.synchronize()
     _check_status(s)
     kt = s.ctx.kernel_times(reset=True)
-    assert kt["prefill_pair_tcgen05" if rows == 256 else "dense_tcgen05"][1] == 2
+    assert kt["prefill_pair_tcgen05" if rows == 256 else "dense_tcgen05"][1] == (1 if only_reloading else 2)
     row = 0
     for r, off, c in chunks:
         o_ref, l_ref = oracle.workload_prefill_chunk(w, t, r, off, c)
