@@ -169,6 +169,35 @@ def test_capacity_limits(lib):
     assert e.value.code == B.TPA_ERR_CAPACITY
 
 
+def test_degenerate_batches_are_refused_and_leave_tables_unchanged(lib):
+    ctx = plan_ctx(num_pages=100, reqs=4, tokens=64)
+    ctx.prefix_register(0, 40)
+    for r in range(3):
+        ctx.request_open(r, 0)
+    ctx.kv_append([0, 1, 2], [5, 17, 1], 1, 1)
+    lens = [ctx.query(B.Q_SUFFIX_LEN, r) for r in range(3)]
+    free = ctx.query(B.Q_FREE_PAGES)
+    cases = [
+        (lambda: ctx.decode([], 1, 1, 1, 1, 1), B.TPA_ERR_INVALID_ARG),              # empty batch
+        (lambda: ctx.prefill_chunk([], [], 1, 1, 1, 1, 1), B.TPA_ERR_INVALID_ARG),
+        (lambda: ctx.kv_append([], [], 1, 1), B.TPA_ERR_INVALID_ARG),
+        (lambda: ctx.decode([0, 1, 0], 1, 1, 1, 1, 1), B.TPA_ERR_INVALID_ARG),       # a request twice
+        (lambda: ctx.prefill_chunk([1, 1], [4, 4], 1, 1, 1, 1, 1), B.TPA_ERR_INVALID_ARG),
+        (lambda: ctx.prefill_chunk([0, 1], [4, 0], 1, 1, 1, 1, 1), B.TPA_ERR_INVALID_ARG),  # empty chunk
+        (lambda: ctx.decode([0, 4], 1, 1, 1, 1, 1), B.TPA_ERR_INVALID_ARG),          # id out of range
+        (lambda: ctx.decode([0, -1], 1, 1, 1, 1, 1), B.TPA_ERR_INVALID_ARG),
+        (lambda: ctx.decode([0, 3], 1, 1, 1, 1, 1), B.TPA_ERR_STATE),                # not open
+    ]
+    for call, code in cases:
+        with pytest.raises(B.TpaError) as e:
+            call()
+        assert e.value.code == code
+        assert [ctx.query(B.Q_SUFFIX_LEN, r) for r in range(3)] == lens
+        assert ctx.query(B.Q_FREE_PAGES) == free
+    ctx.decode([0, 1, 2], 1, 1, 1, 1, 1)         # and the context still works
+    assert [ctx.query(B.Q_SUFFIX_LEN, r) for r in range(3)] == [n + 1 for n in lens]
+
+
 def test_decode_plan_decomposition(lib):
     """Llama-3-8B decode shape: 4 agents x 4096-token prefixes, 16 requests each."""
     hq, hkv, G = 32, 8, 4
