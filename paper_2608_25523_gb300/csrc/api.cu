@@ -793,9 +793,10 @@ int tpa_prefix_reload(tpa_ctx* ctx, int32_t agent, const void* host_k, const voi
   if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
   if (a.resident) return fail(TPA_ERR_STATE, "agent %d is already resident", agent);
   if (a.len > 0 && (!host_k || !host_v)) return fail(TPA_ERR_INVALID_ARG, "null source");
-  const void* kd = host_k;
-  const void* vd = host_v;
   if (!ctx->plan_only && a.len > 0) {
+    // the copy engine reads the source: pinned host (or device) memory only
+    const void* kd;
+    const void* vd;
     int rc;
     if ((rc = resolve_host_ptr(host_k, &kd)) || (rc = resolve_host_ptr(host_v, &vd))) return rc;
   }
@@ -829,9 +830,10 @@ int tpa_prefix_offload(tpa_ctx* ctx, int32_t agent, void* host_k, void* host_v, 
   if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
   if (!a.resident) return fail(TPA_ERR_NOT_RESIDENT, "agent %d is not resident", agent);
   if (a.len > 0 && (!host_k || !host_v)) return fail(TPA_ERR_INVALID_ARG, "null destination");
-  const void* kd = host_k;
-  const void* vd = host_v;
   if (!ctx->plan_only && a.len > 0) {
+    // the copy engine writes the destination: pinned host (or device) memory only
+    const void* kd;
+    const void* vd;
     int rc;
     if ((rc = resolve_host_ptr(host_k, &kd)) || (rc = resolve_host_ptr(host_v, &vd))) return rc;
   }
