@@ -729,6 +729,12 @@ def bench_movement(args, dev):
             ov[:ell].copy_(dk[:ell], non_blocking=True)
 
         with torch.cuda.stream(side):
+            # the page kernel on the mapped host arrays (TPA_OPT_MOVEMENT_STAGED 0) ...
+            ctx.set_option(B.OPT_MOVEMENT_STAGED, 0)
+            t_re_d = timed(reload, before=evict)
+            t_off_d = timed(offload, before=make_resident)
+            # ... and the default: copy engine through the staging area
+            ctx.set_option(B.OPT_MOVEMENT_STAGED, 1)
             t_re = timed(reload, before=evict)
             t_off = timed(offload, before=make_resident)
             side.synchronize()
@@ -737,7 +743,8 @@ def bench_movement(args, dev):
             t_h2d, t_d2h = timed(h2d), timed(d2h)
         side.synchronize()
         rows.append({"tokens": ell, "bytes": ell * mu, "reload_us": round(t_re, 1),
-                     "offload_us": round(t_off, 1), "h2d_copy_us": round(t_h2d, 1),
+                     "offload_us": round(t_off, 1), "reload_direct_us": round(t_re_d, 1),
+                     "offload_direct_us": round(t_off_d, 1), "h2d_copy_us": round(t_h2d, 1),
                      "d2h_copy_us": round(t_d2h, 1), "round_trip_bit_exact": exact})
         evict()
 
@@ -753,6 +760,7 @@ def bench_movement(args, dev):
     res = {"workload": "prefix movement, llama3_8b layer (mu = 4096 B/token), prefixes of "
                        + ", ".join(str(x) for x in sizes) + " tokens, permuted pool",
            "rows": rows, "reload": fit("reload_us"), "offload": fit("offload_us"),
+           "reload_direct": fit("reload_direct_us"), "offload_direct": fit("offload_direct_us"),
            "h2d_copy": fit("h2d_copy_us"), "d2h_copy": fit("d2h_copy_us")}
     res["mu_over_B_swap_ns_per_token"] = {
         "reload": round(mu / (res["reload"]["B_gbs"] * 1e9) * 1e9, 3),

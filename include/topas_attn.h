@@ -278,6 +278,11 @@ enum {
                                    tile (one CTA, two softmax warpgroups, the tensor pipe
                                    alternating between them); 128 runs single tiles through the
                                    dense kernel of the decode's level 1 */
+  TPA_OPT_MOVEMENT_STAGED = 8,  /* prefix reload / offload: 1 (default) moves the prefix over the
+                                   host link with the copy engine, through the workspace's
+                                   staging area, and scatters / gathers the pages on the device;
+                                   0 runs the page kernel on the mapped host arrays directly (it
+                                   holds its SMs for the whole link-bound transfer) */
 };
 TPA_API int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value);
 

@@ -38,6 +38,7 @@ OPT_KERNEL_TIMING = 4
 OPT_TEST_PLAN_WAIT = 5
 OPT_PREFILL_TILE_ROWS = 6
 OPT_TEST_BAD_PAGE = 7
+OPT_MOVEMENT_STAGED = 8
 # kernel kinds of tpa_kernel_times
 KERNEL_NAMES = ["kv_append", "dense_tcgen05", "split_kv", "lse_merge", "page_copy",
                 "prefill_pair_tcgen05"]

@@ -164,7 +164,8 @@ struct tpa_ctx {
 
   // options and statistics
   int decode_mode = 0;
-  int prefill_rows = 256;  // query rows per prefill work item: 256 (tile pairs) or 128
+  int prefill_rows = 256;
+  bool staged_movement = true;  // TPA_OPT_MOVEMENT_STAGED  // query rows per prefill work item: 256 (tile pairs) or 128
   int test_plan_wait = 0;  // test hook: the next cascade decode waits for a flag never written
   int test_bad_page = 0;   // test hook: the next decode's first prefix page id is out of the pool
   int prefix_splits = 0;
@@ -793,13 +794,15 @@ int tpa_prefix_reload(tpa_ctx* ctx, int32_t agent, const void* host_k, const voi
   if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
   if (a.resident) return fail(TPA_ERR_STATE, "agent %d is already resident", agent);
   if (a.len > 0 && (!host_k || !host_v)) return fail(TPA_ERR_INVALID_ARG, "null source");
+  // pinned host (or device) memory only; the direct mode's kernel reads it
+  // through its mapped device address
+  const void* kd = host_k;
+  const void* vd = host_v;
   if (!ctx->plan_only && a.len > 0) {
-    // the copy engine reads the source: pinned host (or device) memory only
-    const void* kd;
-    const void* vd;
     int rc;
     if ((rc = resolve_host_ptr(host_k, &kd)) || (rc = resolve_host_ptr(host_v, &vd))) return rc;
   }
+  const bool staged = ctx->staged_movement;
   const int64_t need = cdiv(a.len, kPage);
   if (need > free_count(ctx))
     return fail(TPA_ERR_NO_SPACE, "reload needs %lld pages, %lld free", (long long)need,
@@ -807,8 +810,9 @@ int tpa_prefix_reload(tpa_ctx* ctx, int32_t agent, const void* host_k, const voi
   std::vector<int32_t> pages;
   const uint64_t tag = take_pages(ctx, need, pages);
   cudaStream_t s = static_cast<cudaStream_t>(side_stream);
-  const int rc = page_copy_call(ctx, pages, a.len, 1, host_k, host_v, nullptr, nullptr, s, false,
-                                std::max(tag, a.last_use), nullptr, true);
+  const int rc = page_copy_call(ctx, pages, a.len, 1, staged ? host_k : kd, staged ? host_v : vd,
+                                nullptr, nullptr, s, false, std::max(tag, a.last_use), nullptr,
+                                staged);
   if (rc) {
     // give the pages back untouched (nothing was queued that writes them)
     for (auto it = pages.rbegin(); it != pages.rend(); ++it) ctx->free_pages[--ctx->free_head] = *it;
@@ -830,18 +834,22 @@ int tpa_prefix_offload(tpa_ctx* ctx, int32_t agent, void* host_k, void* host_v, 
   if (a.len < 0) return fail(TPA_ERR_STATE, "agent %d is not registered", agent);
   if (!a.resident) return fail(TPA_ERR_NOT_RESIDENT, "agent %d is not resident", agent);
   if (a.len > 0 && (!host_k || !host_v)) return fail(TPA_ERR_INVALID_ARG, "null destination");
+  // pinned host (or device) memory only; the direct mode's kernel writes it
+  // through its mapped device address
+  const void* kd = host_k;
+  const void* vd = host_v;
   if (!ctx->plan_only && a.len > 0) {
-    // the copy engine writes the destination: pinned host (or device) memory only
-    const void* kd;
-    const void* vd;
     int rc;
     if ((rc = resolve_host_ptr(host_k, &kd)) || (rc = resolve_host_ptr(host_v, &vd))) return rc;
   }
+  const bool staged = ctx->staged_movement;
   cudaStream_t s = static_cast<cudaStream_t>(side_stream);
   // the pages' last writer/readers must finish before the copy reads them
   wait_for_seq(ctx, ctx->chain_seq, s);
-  const int rc = page_copy_call(ctx, a.pages, a.len, 0, nullptr, nullptr, host_k, host_v, s, false,
-                                std::max(a.ready_seq, a.last_use), nullptr, true);
+  const int rc = page_copy_call(ctx, a.pages, a.len, 0, nullptr, nullptr,
+                                staged ? host_k : const_cast<void*>(kd),
+                                staged ? host_v : const_cast<void*>(vd), s, false,
+                                std::max(a.ready_seq, a.last_use), nullptr, staged);
   if (rc) return rc;
   a.last_use = ctx->seq;
   give_pages(ctx, a.pages, ctx->seq);
@@ -1697,6 +1705,9 @@ int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
       return TPA_OK;
     case TPA_OPT_TEST_BAD_PAGE:
       ctx->test_bad_page = value ? 1 : 0;
+      return TPA_OK;
+    case TPA_OPT_MOVEMENT_STAGED:
+      ctx->staged_movement = value != 0;
       return TPA_OK;
     case TPA_OPT_PREFILL_TILE_ROWS:
       if (value != 128 && value != 256) return fail(TPA_ERR_INVALID_ARG, "prefill tile rows %lld", (long long)value);

@@ -216,10 +216,14 @@ def test_page_roundtrip_bit_exact(perm):
     _check_status(s)
 
 
-def test_offload_reload_bit_exact_on_side_stream():
+@pytest.mark.parametrize("staged", [1, 0], ids=["staged", "direct"])
+def test_offload_reload_bit_exact_on_side_stream(staged):
+    """Both movement modes: copy engine through the staging area (default)
+    and the page kernel on the mapped host arrays."""
     w = small_case(23, hq=8, hkv=2, d=128, prefix_len=[333, 48], req_agent=[0, 1, 0],
                    req_ctx=[20, 5, 77], req_prefill=[0] * 3, req_decode=[1] * 3, permute=True)
     t, s = _session(w)
+    s.ctx.set_option(B.OPT_MOVEMENT_STAGED, staged)
     L = w.prefix_len[0]
     hk = torch.empty(L, 2, 128, dtype=torch.bfloat16, pin_memory=True)
     hv = torch.empty_like(hk, pin_memory=True)
