@@ -17,7 +17,7 @@ import oracle
 from paper_2608_25523_gb300 import binding as B
 from paper_2608_25523_gb300.build import build
 from paper_2608_25523_gb300.session import Session, to_device
-from paper_2608_25523_gb300.workloads import config, sharp, small_case, tensors_numpy
+from paper_2608_25523_gb300.workloads import bf16_round, config, sharp, small_case, tensors_numpy
 
 from _util import compare, stack_decode_ref
 
@@ -157,6 +157,31 @@ def test_prefill_chunks(name, rows):
             o_ref, l_ref = oracle.workload_prefill_chunk(w, t, r, off, c)
             compare(out[row:row + c], lse[row:row + c], o_ref, l_ref, f"{name} r{r} off{off}")
             row += c
+
+
+@pytest.mark.parametrize("rows", [256, 128], ids=["pairs", "single"])
+def test_prefill_scores_rising_far_above_the_first_tile(rows):
+    """Suffix keys 24x larger than the prefix keys: the scores of the
+    suffix tiles lie far above the prefix tiles' row max, so the online
+    softmax's reference max jumps by tens of log2 units mid-row and O and l
+    are rescaled.  The outputs must still match the oracle."""
+    w = small_case(41, hq=8, hkv=2, d=128, prefix_len=[300, 150], req_agent=[0, 1, 0],
+                   req_ctx=[0] * 3, req_prefill=[200, 130, 64], req_decode=[0] * 3, chunk=256,
+                   permute=True)
+    t = tensors_numpy(w)
+    t.suffix_k = bf16_round(t.suffix_k * np.float32(24.0))
+    s = Session(w, to_device(t, "cuda"))
+    s.ctx.set_option(B.OPT_PREFILL_TILE_ROWS, rows)
+    chunks, ids, lens, q, k, v = s.prefill_inputs(0)
+    out, lse = s.new_outputs(sum(lens))
+    s.prefill(ids, lens, q, k, v, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    row = 0
+    for r, off, c in chunks:
+        o_ref, l_ref = oracle.workload_prefill_chunk(w, t, r, off, c)
+        compare(out[row:row + c], lse[row:row + c], o_ref, l_ref, f"r{r} off{off}")
+        row += c
 
 
 def test_tiny_workload_prefill_then_decode():
