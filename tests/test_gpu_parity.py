@@ -94,6 +94,27 @@ def test_decode_split_choices_agree(splits):
     compare(out, lse, o_ref, l_ref, f"splits {splits}")
 
 
+@pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
+def test_decode_suffix_scores_far_above_the_prefix(mode):
+    """Suffix keys 24x larger than the prefix keys: the partials of one
+    token have LSEs tens of units apart, so the exact merge must weight the
+    prefix partials down to (almost) nothing.  Must match the oracle."""
+    w = small_case(43, hq=8, hkv=2, d=128, prefix_len=[700, 129], req_agent=[0, 1, 0, 1, 0],
+                   req_ctx=[40, 300, 1, 17, 600], req_prefill=[0] * 5, req_decode=[1] * 5,
+                   permute=True)
+    t = tensors_numpy(w)
+    t.suffix_k = bf16_round(t.suffix_k * np.float32(24.0))
+    s = Session(w, to_device(t, "cuda"))
+    s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "suffix scores far above the prefix")
+
+
 def test_decode_sharp_softmax():
     w = sharp(small_case(11, hq=8, hkv=2, d=128, prefix_len=[513, 64], req_agent=[0, 1, 0, 1, 0],
                          req_ctx=[40, 2, 129, 300, 0], req_prefill=[0] * 5, req_decode=[1] * 5))
