@@ -184,10 +184,12 @@ TPA_API int tpa_kv_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const in
  * sees all ell_a prefix keys and suffix positions 0..p (diagonal
  * included).
  *   chunk_len[i] (host): tokens in request i's chunk (>= 1)
- *   q      device bf16 [sum chunk_len][Hq][d]
- *   k_new  device bf16 [sum chunk_len][Hkv][d]   (v_new likewise)
- *   out    device bf16 [sum chunk_len][Hq][d]
- *   lse    device fp32 [sum chunk_len][Hq]  natural-log LSE of the scaled scores
+ *   q      bf16 [sum chunk_len][Hq][d]
+ *   k_new  bf16 [sum chunk_len][Hkv][d]   (v_new likewise)
+ *   out    bf16 [sum chunk_len][Hq][d]
+ *   lse    fp32 [sum chunk_len][Hq]  natural-log LSE of the scaled scores
+ * Device memory, or pinned host memory as for tpa_decode (the kernels then
+ * move those bytes over the CPU-GPU link; the results are bit-identical).
  * Errors: INVALID_ARG, STATE, NOT_RESIDENT, NO_SPACE, CAPACITY, CUDA. */
 TPA_API int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* chunk_len,
                       const void* q, const void* k_new, const void* v_new,

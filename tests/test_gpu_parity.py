@@ -329,6 +329,29 @@ def test_decode_with_pinned_host_io_is_bit_identical():
     compare(ho, hl, o_ref, l_ref, "pinned host io")
 
 
+@pytest.mark.parametrize("rows", [256, 128], ids=["pairs", "single"])
+def test_prefill_with_pinned_host_io_is_bit_identical(rows):
+    """A prefill chunk round with q, k_new, v_new, out, lse in pinned host
+    memory gives the same bits as with device buffers."""
+    w = small_case(47, hq=8, hkv=2, d=128, prefix_len=[300, 17], req_agent=[0, 1, 0],
+                   req_ctx=[0] * 3, req_prefill=[100, 64, 37], req_decode=[0] * 3, chunk=128,
+                   permute=True)
+    t, s = _session(w)
+    s.ctx.set_option(B.OPT_PREFILL_TILE_ROWS, rows)
+    chunks, ids, lens, q, k, v = s.prefill_inputs(0)
+    out, lse = s.new_outputs(sum(lens))
+    s.prefill(ids, lens, q, k, v, out, lse)
+    s.ctx.request_truncate(ids, [0] * len(ids))
+    pin = lambda x: x.cpu().pin_memory()
+    hq, hk, hv = pin(q), pin(k), pin(v)
+    ho = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+    hl = torch.empty(lse.shape, dtype=lse.dtype, pin_memory=True)
+    s.prefill(ids, lens, hq, hk, hv, ho, hl)
+    torch.cuda.synchronize()
+    _check_status(s)
+    assert torch.equal(_bits(ho), _bits(out.cpu())) and torch.equal(hl, lse.cpu())
+
+
 def test_concurrent_reloads_on_two_streams_share_the_staging_area():
     """Two prefixes reloaded at once on two side streams go through the one
     staging area of the workspace; the second waits for the first on the
