@@ -1444,7 +1444,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   std::vector<int32_t> agents_seen;
   PlanSizes sz;
   sz.append = total;
-  sz.dense_tok = total;
+  sz.dense_tok = pairs ? 0 : total;  // paired items derive their tokens from row0 / pos0
   std::unordered_map<int32_t, int32_t> agent_off;
   for (int i = 0; i < n; ++i) {
     const int32_t a = ctx->reqs[reqs[i]].agent;
@@ -1516,11 +1516,16 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
     const int c = chunk_len[i];
     for (int t0 = 0; t0 < c; t0 += tpt) {
       const int t1 = std::min(c, t0 + tpt);
-      const int32_t tok_base = nt;
-      for (int t = t0; t < t1; ++t)
-        w.dtok[nt++] = DenseTok{static_cast<int32_t>(row0 + t), offset[i] + t, 0, 0};
       DenseItem it{};
-      it.tok_base = tok_base;
+      if (pairs) {
+        it.tok_base = -1;
+        it.row0 = static_cast<int32_t>(row0 + t0);
+        it.pos0 = offset[i] + t0;
+      } else {
+        it.tok_base = nt;
+        for (int t = t0; t < t1; ++t)
+          w.dtok[nt++] = DenseTok{static_cast<int32_t>(row0 + t), offset[i] + t, 0, 0};
+      }
       it.n_tok = t1 - t0;
       it.out_mode = 1;
       it.seg_pages[0] = agent_off[r.agent];

@@ -274,12 +274,17 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
       return false;
     };
     constexpr DenseTok kNoTok = {0, 0x7fffffff, 0, 0};
+    // token i of an item: its DenseTok record, or derived from the item
+    // (consecutive rows of one chunk)
+    auto tok_of = [&](const DenseItem& it, int i) {
+      return it.tok_base >= 0 ? p.toks[it.tok_base + i] : DenseTok{it.row0 + i, it.pos0 + i, 0, 0};
+    };
     // this thread's Q row of an item (zero for rows past the item's tokens),
     // into the swizzled Q tile
     auto load_q = [&](const DenseItem& it) {
       const bool valid = tok_in < it.n_tok;
       const int head = it.kv_head * G + row % G;
-      const DenseTok t = valid ? p.toks[it.tok_base + tok_in] : kNoTok;
+      const DenseTok t = valid ? tok_of(it, tok_in) : kNoTok;
       const __nv_bfloat16* src =
           p.q + (valid ? (static_cast<int64_t>(t.q_row) * p.hq + head) * D : 0);
 #pragma unroll
@@ -305,7 +310,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
       const int idx_n = item_of(k + 1, n_ctas);
       const bool has_next = idx_n < p.n_items;
       const bool row_valid = tok_in < item.n_tok;
-      const DenseTok dt = row_valid ? p.toks[item.tok_base + tok_in] : kNoTok;
+      const DenseTok dt = row_valid ? tok_of(item, tok_in) : kNoTok;
       const int head = item.kv_head * G + row % G;
       float m_run = -INFINITY, l_run = 0.f;
       bool q_issued = false;

@@ -35,7 +35,7 @@ struct DenseTok {
 // One 128-row query tile (128/G tokens x G heads of one kv head) against up
 // to two key segments, each a run of pages of one prefix or one suffix.
 struct DenseItem {
-  int32_t tok_base;       // first DenseTok of the tile
+  int32_t tok_base;       // first DenseTok of the tile (< 0: consecutive tokens, below)
   int32_t n_tok;          // tokens in the tile (<= 128 / G)
   int32_t kv_head;
   int32_t split;          // split index for partial slots (out_mode 0)
@@ -45,7 +45,11 @@ struct DenseItem {
   int32_t seg_k0[2];      // first key of the range (multiple of 16)
   int32_t seg_k1[2];      // one past the last key of the range (k1 == k0: empty)
   int32_t seg_causal[2];  // 1: causal mask on this segment
-  int32_t pad[2];
+  // tok_base < 0 (paired prefill items): the tile's tokens are consecutive
+  // rows of one chunk, token i at q row row0 + i and causal position pos0 + i,
+  // with no DenseTok records
+  int32_t row0;
+  int32_t pos0;
 };
 static_assert(sizeof(DenseItem) == 64, "DenseItem layout");
 
