@@ -930,14 +930,29 @@ static int reserve_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const in
   return TPA_OK;
 }
 
+// Runs (one per page touched) of appending ntok[i] tokens after each
+// request's current length: the count, and the records themselves (source
+// rows follow the requests' order).
+static int64_t append_runs(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* ntok) {
+  int64_t runs = 0;
+  for (int i = 0; i < n; ++i)
+    if (ntok[i] > 0) runs += cdiv(ctx->reqs[reqs[i]].len % kPage + ntok[i], kPage);
+  return runs;
+}
+
 static void write_append_rows(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* ntok,
                               AppendRow* rows) {
-  int64_t row = 0;
+  int64_t run = 0;
+  int32_t src = 0;
   for (int i = 0; i < n; ++i) {
     const Request& r = ctx->reqs[reqs[i]];
-    for (int t = 0; t < ntok[i]; ++t, ++row) {
+    for (int t = 0; t < ntok[i];) {
       const int pos = r.len + t;
-      rows[row] = AppendRow{static_cast<int32_t>(row), r.pages[pos / kPage], pos % kPage, 0};
+      const int slot = pos % kPage;
+      const int cnt = std::min(kPage - slot, ntok[i] - t);
+      rows[run++] = AppendRow{src, r.pages[pos / kPage], slot, cnt};
+      src += cnt;
+      t += cnt;
     }
   }
 }
@@ -957,10 +972,11 @@ int tpa_kv_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* n
   Slot* sl = acquire_slot(ctx);
   ++ctx->seq;
   PlanSizes sz;
-  sz.append = total;
+  const int64_t runs = append_runs(ctx, n, reqs, ntok);
+  sz.append = runs;
   const PlanLayout lay = layout_of(sz);
   PlanWriter w(sl->host, lay);
-  w.hdr->n_append = static_cast<int32_t>(total);
+  w.hdr->n_append = static_cast<int32_t>(runs);
   write_append_rows(ctx, n, reqs, ntok, w.append);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   chain_begin(ctx, s);
@@ -968,7 +984,7 @@ int tpa_kv_append(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_t* n
   if ((rc = upload(ctx, sl, lay.total, s))) return rc;
   if (!ctx->plan_only) {
     KernelTimer kt(ctx, K_APPEND, s);
-    CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
+    CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(runs), k_new,
                            v_new, ctx->pool, ctx->status, s));
   }
   for (int i = 0; i < n; ++i) {
@@ -1025,7 +1041,7 @@ static DenseParams dense_params(tpa_ctx* ctx, const Slot* sl, const PlanLayout& 
 //  cascade (default): one persistent tcgen05 launch.  Work items are the
 //    stacked shared-prefix tiles of each agent (level 1) and, per token and
 //    kv head, its suffix (level 2, which also appends the step's token);
-//    the last partial of each (token, kv head) triggers the in-kernel merge.
+//    then the LSE merge, launched as its programmatic dependent.
 //  flat (cross-check): KV append, the split-KV kernel over every key of
 //    each request (prefix included), and a separate LSE merge.
 int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, const void* k_new,
@@ -1443,7 +1459,8 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
 
   std::vector<int32_t> agents_seen;
   PlanSizes sz;
-  sz.append = total;
+  const int64_t runs = append_runs(ctx, n, reqs, chunk_len);
+  sz.append = runs;
   sz.dense_tok = pairs ? 0 : total;  // paired items derive their tokens from row0 / pos0
   std::unordered_map<int32_t, int32_t> agent_off;
   for (int i = 0; i < n; ++i) {
@@ -1471,17 +1488,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
     std::memcpy(w.pages + np, ag.pages.data(), ag.pages.size() * 4);
     np += static_cast<int32_t>(ag.pages.size());
   }
-  // append rows use the positions before this call
-  {
-    int64_t row = 0;
-    for (int i = 0; i < n; ++i) {
-      const Request& r = ctx->reqs[reqs[i]];
-      for (int t = 0; t < chunk_len[i]; ++t, ++row) {
-        const int pos = offset[i] + t;
-        w.append[row] = AppendRow{static_cast<int32_t>(row), r.pages[pos / kPage], pos % kPage, 0};
-      }
-    }
-  }
+  write_append_rows(ctx, n, reqs, chunk_len, w.append);  // positions before this call
   // Items go straight to their place, the early chunks' items first, each
   // group in longest-first order (a stable counting sort on the key-tile
   // count): first count the items of each length, then write them.
@@ -1549,7 +1556,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   }
   PlanHeader* hd = w.hdr;
   hd->n_pages = np;
-  hd->n_append = static_cast<int32_t>(total);
+  hd->n_append = static_cast<int32_t>(runs);
   hd->n_dense_tok = nt;
   hd->n_dense = nd;
 
@@ -1559,7 +1566,7 @@ int tpa_prefill_chunk(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const int32_
   if (!ctx->plan_only) {
     {
       KernelTimer kt(ctx, K_APPEND, s);
-      CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(total), k_new,
+      CUDA_TRY(launch_append(dev_ptr<AppendRow>(sl, lay.off_append), static_cast<int>(runs), k_new,
                              v_new, ctx->pool, ctx->status, s));
     }
     // items [0, n_early) after the reloads of their agents (if any is

@@ -24,16 +24,17 @@ constexpr int kCopyThreads = 256;
 constexpr int kAppendUnroll = 4;
 
 // Unit x of the call (32-bit: the host checks the count) is 16-byte unit
-// x % upr of row x / upr, where a row is one token's K (or V) across the kv
-// heads; each thread loads kAppendUnroll units of K and of V before it
+// x % upr of slot (x / upr) % 16 of run x / (16 upr), where a slot row is
+// one token's K (or V) across the kv heads and slots past the run's n are
+// idle; each thread loads kAppendUnroll units of K and of V before it
 // stores any, so enough bytes are in flight to stream at HBM rate.
 template <int CPR>
 __global__ void __launch_bounds__(kCopyThreads)
-    append_kernel(const AppendRow* __restrict__ rows, int n_rows, const uint4* __restrict__ k_src,
+    append_kernel(const AppendRow* __restrict__ rows, int n_runs, const uint4* __restrict__ k_src,
                   const uint4* __restrict__ v_src, uint4* __restrict__ k_pool,
                   uint4* __restrict__ v_pool, int64_t num_pages, int hkv, uint32_t* status) {
   const int upr = hkv * CPR;
-  const int total = n_rows * upr;
+  const int total = n_runs * kPage * upr;
   const int stride = gridDim.x * blockDim.x;
   for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < total; u += kAppendUnroll * stride) {
     uint4 kx[kAppendUnroll], vx[kAppendUnroll];
@@ -43,16 +44,18 @@ __global__ void __launch_bounds__(kCopyThreads)
       dst[i] = -1;
       const int x = u + i * stride;
       if (x >= total) continue;
-      const int row = x / upr;
+      const int row = x / upr;  // run * 16 + token of the run
       const int rem = x - row * upr;
-      const AppendRow r = rows[row];
-      if (r.page < 0 || r.page >= num_pages || r.slot < 0 || r.slot >= kPage) {
+      const AppendRow r = rows[row / kPage];
+      const int j = row % kPage;
+      if (j >= r.n) continue;
+      if (r.page < 0 || r.page >= num_pages || r.slot < 0 || r.slot + r.n > kPage) {
         atomicOr(status, kStatusBadPage);
         continue;
       }
       const int h = rem / CPR, c = rem % CPR;
-      dst[i] = ((static_cast<int64_t>(r.page) * hkv + h) * kPage + r.slot) * CPR + c;
-      const int64_t src = static_cast<int64_t>(r.src) * upr + rem;
+      dst[i] = ((static_cast<int64_t>(r.page) * hkv + h) * kPage + r.slot + j) * CPR + c;
+      const int64_t src = static_cast<int64_t>(r.src + j) * upr + rem;
       kx[i] = k_src[src];
       vx[i] = v_src[src];
     }
@@ -104,12 +107,12 @@ int copy_grid(int64_t units) {
 
 }  // namespace
 
-cudaError_t launch_append(const AppendRow* rows, int n_rows, const void* k_src,
+cudaError_t launch_append(const AppendRow* rows, int n_runs, const void* k_src,
                           const void* v_src, const PoolGeom& pool, uint32_t* status,
                           cudaStream_t stream) {
-  if (n_rows <= 0) return cudaSuccess;
+  if (n_runs <= 0) return cudaSuccess;
   const int cpr = pool.d / 8;
-  const int64_t units = static_cast<int64_t>(n_rows) * pool.hkv * cpr;
+  const int64_t units = static_cast<int64_t>(n_runs) * kPage * pool.hkv * cpr;
   if (units > INT32_MAX || (cpr != 8 && cpr != 16)) return cudaErrorInvalidValue;
   const int grid = copy_grid((units + kAppendUnroll - 1) / kAppendUnroll);
   auto* const ks = static_cast<const uint4*>(k_src);
@@ -117,10 +120,10 @@ cudaError_t launch_append(const AppendRow* rows, int n_rows, const void* k_src,
   auto* const kp = static_cast<uint4*>(pool.k);
   auto* const vp = static_cast<uint4*>(pool.v);
   if (cpr == 16)
-    append_kernel<16><<<grid, kCopyThreads, 0, stream>>>(rows, n_rows, ks, vs, kp, vp,
+    append_kernel<16><<<grid, kCopyThreads, 0, stream>>>(rows, n_runs, ks, vs, kp, vp,
                                                          pool.num_pages, pool.hkv, status);
   else
-    append_kernel<8><<<grid, kCopyThreads, 0, stream>>>(rows, n_rows, ks, vs, kp, vp,
+    append_kernel<8><<<grid, kCopyThreads, 0, stream>>>(rows, n_runs, ks, vs, kp, vp,
                                                         pool.num_pages, pool.hkv, status);
   return cudaGetLastError();
 }

@@ -18,9 +18,9 @@ struct PoolGeom {
   int d;
 };
 
-// K/V writes: one row per token into (page, slot).  k_src/v_src are
-// [rows][hkv][d]; device or mapped pinned-host pointers.
-cudaError_t launch_append(const AppendRow* rows, int n_rows, const void* k_src,
+// K/V writes: `n_runs` runs of consecutive tokens, each within one page.
+// k_src/v_src are [tokens][hkv][d]; device or mapped pinned-host pointers.
+cudaError_t launch_append(const AppendRow* rows, int n_runs, const void* k_src,
                           const void* v_src, const PoolGeom& pool, uint32_t* status,
                           cudaStream_t stream);
 

@@ -15,13 +15,13 @@ constexpr uint32_t kStatusSuffixTimeout = 2u;
 constexpr uint32_t kStatusBadPage = 4u;
 constexpr uint32_t kStatusPlanTimeout = 8u;  // a plan upload never arrived
 
-// One token row of a KV write: row `src` of the source K/V arrays goes to
-// slot `slot` of page `page`.
+// A run of a KV write within one page: source rows src .. src + n - 1 of
+// the K/V arrays go to slots slot .. slot + n - 1 of page `page` (n <= 16).
 struct AppendRow {
   int32_t src;
   int32_t page;
   int32_t slot;
-  int32_t pad;
+  int32_t n;
 };
 
 // Per-token data of a dense tile.
