@@ -1,34 +1,44 @@
 """Benchmark of shared-prefix paged attention on one GB300 (or N replicas).
 
-Default workload: the Llama-3-8B attention layer decode step (32 q heads,
-8 kv heads, head_dim 128, bf16): 4 agents with 4096-token prefixes, 64
-decode requests (16 per agent) with cached suffixes uniform in 256..1024,
-page size 16.  One step = one tpa_decode call over the 64 requests (host plan,
-one upload, one persistent tcgen05 launch that appends the new tokens and
-runs the stacked shared-prefix tiles and the per-request suffixes, and the
-log-sum-exp merge launched as its programmatic dependent), followed by a
-table-only truncate that drops
-the appended token again so every step sees the same workload.  Four
-independent copies of the workload are cycled so that ~0.94 GB of KV lies
-between two visits of the same bytes (L2 is 129 MB): every step reads HBM.
+Headline workload: the Llama-3-70B attention layer decode step (64 q heads,
+8 kv heads, head_dim 128, bf16): 6 agents with 16384-token prefixes, 512
+decode requests (86,86,85,85,85,85) with cached suffixes uniform in
+512..4096, page size 16, contiguous pages; 5.35 GB of KV per layer.  The
+workload is sized to fill most of a 180 GB HBM: L layer pools (26 by
+default, one context each, the same page and request tables, each with its
+own seeded KV and queries), 157 GB resident.  One step = one tpa_decode
+call per layer, layer after layer, as a model's forward pass makes them
+(host plan, one upload, one persistent tcgen05 launch that appends the new
+tokens and runs the stacked shared-prefix tiles and the per-request
+suffixes, and the log-sum-exp merge launched as its programmatic
+dependent), each followed by a table-only truncate that drops the appended
+token again so every step sees the same workload.  Consecutive decodes
+never share an L2-resident byte (each layer's KV is 41x the L2).
 
-value  = algorithmic bytes per step (each prefix once, each suffix once,
-         Q, the new tokens' K/V in and out, O and LSE) / device time, GB/s.
-e2e    = the same metric through the public call with host buffers: the
-         step's q / k_new / v_new sit in pinned host memory and O / LSE go
-         back to it, inside the timed region.  tpa_decode takes the host
+value  = algorithmic bytes per step (per layer: each prefix once, each
+         suffix once, Q, the new tokens' K/V in and into the pool, O and
+         LSE; times L) / device time, GB/s.
+e2e    = the same metric through the public call with host buffers: each
+         layer's q / k_new / v_new sit in pinned host memory and its O / LSE
+         go back to it, inside the timed region.  tpa_decode takes the host
          arrays themselves and its kernels move those bytes over the
          CPU-GPU link; the variant with copy-engine copies to and from
          device buffers is reported beside it (e2e.copy_engine).
-Also reported (rank 0, N=1): the tcgen05 chunked-prefill workload
-(TFLOP/s), the mixed workload (reload + prefill + Zipf decode, ms/step),
-the Llama-3-70B decode workload (GB/s), each with its own roofline, the
-prefix-movement calibration (reload / offload bandwidth, the paper's
-mu / B_swap), the redo trade of a preempted suffix (decode steps vs
-chunked prefill), a kernel-level analogue of the paper's co-residency
-diagnostic (one vs two resident prefixes under one KV budget), and the
-TOPAS scheduler driving the library on Chain-3 tasks (decision latency,
-native and oracle).
+
+Also reported (rank 0, N=1), each reduced to its headline fields in the
+printed line (--detail PATH writes everything):
+  decode_8b    the Llama-3-8B layer decode step (4 agents x 4096-token
+               prefixes, 64 requests), 4 copies cycled, its own step count;
+  prefill      the chunked-prefill workload (TFLOP/s, tensor roofline);
+  mixed        reload + prefill + Zipf decode on a fragmented pool (ms/step);
+  movement     prefix reload / offload bandwidth, the paper's mu / B_swap;
+  redo         the redo trade of a preempted suffix (decode steps against
+               chunked prefill);
+  coresidency  a kernel-level analogue of the paper's co-residency
+               diagnostic: admissible batch and tokens/s as the number of
+               co-resident prefixes grows under one KV budget;
+  sched        the TOPAS scheduler driving the library on Chain-3 tasks
+               (decision latency, native and oracle).
 
 Under torchrun every rank runs its own copy on its own GPU (the path has
 no exchange step: replicas only); value aggregates all ranks over the
@@ -53,7 +63,8 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "decode KV HBM GB/s (% of peak) + prefill TFLOP/s, tokens/s at 1×GB300"
-COPIES = 4
+COPIES = 4          # copies of the 8B decode workload cycled to defeat L2
+LAYERS_70B = 26     # layer pools of the 70B workload (5.4 GB of KV each)
 
 
 def peaks():
@@ -66,10 +77,11 @@ def peaks():
 
 # ------------------------------------------------------------ accounting --
 
-# Sources of the unified decode kernel; the DRAM traffic recorded in its ncu
+# Sources of the unified decode kernel; the DRAM traffic recorded in an ncu
 # summary counts only while they are unchanged.
 KERNEL_SOURCES = ["k_dense.cu", "dense_common.cuh", "split_kv.cuh", "ptx.cuh", "plan.h", "kernels.h"]
-PROFILE = os.path.join(ROOT, "profiles", "dense_tcgen05_c2_decode.md")
+PROFILE_8B = os.path.join(ROOT, "profiles", "dense_tcgen05_c2_decode.md")
+PROFILE_70B = os.path.join(ROOT, "profiles", "dense_tcgen05_70b_decode.md")
 
 
 def kernel_source_hash():
@@ -81,12 +93,12 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
+def profiled_traffic(path):
     """DRAM bytes (read + write) per launch of the unified decode kernel from
-    the committed ncu summary, or None if it was taken on other sources."""
+    a committed ncu summary, or None if it was taken on other sources."""
     try:
         vals = {}
-        with open(PROFILE) as fh:
+        with open(path) as fh:
             for line in fh:
                 if ":" in line and line.split(":")[0] in ("traffic_bytes_per_launch",
                                                           "kernel_sources_sha256_16"):
@@ -133,6 +145,20 @@ def job_rate(ms, units_per_rank, world, device):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     return ms, units_per_rank * world / (ms / 1e3)
+
+
+def headline_config(n_layers, world):
+    """`config` of the headline line, shared by both arms."""
+    from paper_2608_25523_gb300.workloads import config
+    w = config(4)
+    layer_bytes = decode_bytes(w, w.decode_requests())[2]
+    return {"workload": f"llama3_70b_decode: Hq64 Hkv8 d128 bf16, 6 x 16384-token prefixes, "
+                        f"512 requests, suffixes U[512,4096], {n_layers} layers",
+            "layers": n_layers,
+            "step": "one decode step of the 512 requests in every layer pool, layer after layer",
+            "l2": "inputs larger than L2: each layer's KV (5.35 GB) is read once per step",
+            "bytes_per_layer": layer_bytes, "bytes_per_step": layer_bytes * n_layers,
+            "parallelism": f"replicas x{world}"}
 
 
 # ---------------------------------------------------------------- clocks --
@@ -188,194 +214,235 @@ class Clocks:
         return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(r[2] for r in inside),
                 "reasons": reasons, "samples": len(inside)}
 
-
 # ------------------------------------------------------------- our arm ---
 
-def run_ours(args, rank, world, local_rank):
+def _packed(tensors, device):
+    """One buffer (pinned when on the host) holding `tensors` back to back,
+    and views of it shaped like them."""
+    import torch
+    sizes = [x.numel() * x.element_size() for x in tensors]
+    buf = torch.empty(sum(sizes), dtype=torch.uint8, device=device, pin_memory=device == "cpu")
+    views, off = [], 0
+    for x, n in zip(tensors, sizes):
+        views.append(buf[off:off + n].view(x.dtype).view(x.shape))
+        off += n
+    return buf, views
+
+
+def build_70b_layers(dev, max_layers):
+    """The 70B decode workload's layer pools: one Session per layer with the
+    same page and request tables and its own seeded KV and queries, as many
+    as fit (at most `max_layers`).  Returns (workload, layers, bytes held
+    per layer, setup seconds); a layer is (session, ids, lens, q, k_new, v_new)."""
+    import dataclasses
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.session import Session
+    from paper_2608_25523_gb300.workloads import config, tensors_torch
+
+    w = config(4)
+    layers = []
+    t0 = time.perf_counter()
+
+    def add_layer(l):
+        wl = w if l == 0 else dataclasses.replace(w, seed=w.seed + 1000 * l)
+        t = tensors_torch(wl, dev)
+        s = Session(wl, t, device=dev, extra_tokens=16, max_tokens=len(w.decode_requests()))
+        ids, q, kn, vn = s.decode_inputs()
+        s.t = None    # the drawn KV now lives in the pool only
+        lens = [w.req_ctx[r] for r in ids]
+        layers.append((s, B.i32_array(ids), B.i32_array(lens), q, kn, vn))
+
+    add_layer(0)
+    torch.cuda.synchronize(dev)
+    s0 = layers[0][0]
+    per_layer = (s0.ctx.k_pool.numel() * 2 * 2 + s0.ctx.workspace.numel()
+                 + 3 * layers[0][3].numel() * 2)
+    free, _ = torch.cuda.mem_get_info(dev)
+    n_layers = max(1, min(max_layers, 1 + int((free - 8e9) // per_layer)))
+    for l in range(1, n_layers):
+        add_layer(l)
+    torch.cuda.synchronize(dev)
+    return w, layers, per_layer, time.perf_counter() - t0
+
+
+def measure_70b(args, rank, world, dev, hbm_peak, peak_src, steps, warmup, with_e2e=True):
+    """The headline: decode steps of the 70B workload over every layer pool.
+
+    Timed region: `steps` steps after `warmup` untimed ones, a barrier and a
+    device synchronize on both sides, CUDA events on the launching stream,
+    nvidia-smi clocks sampled during it (rank 0).  The unified kernel's
+    launches run back to back (the merge of each layer is its programmatic
+    dependent, and the next layer's unified kernel the merge's), so its
+    average launch duration is the timed region over its launches; a short
+    second region with every launch bracketed by events (which breaks that
+    overlap) gives each kernel's share."""
     import torch
     import torch.distributed as dist
-
     from paper_2608_25523_gb300 import binding as B
-    from paper_2608_25523_gb300.build import build
-    from paper_2608_25523_gb300.session import Session
-    from paper_2608_25523_gb300.workloads import config, copy_requests, replicate, tensors_torch
 
-    build()
-    dev = torch.device("cuda", local_rank)
-    torch.cuda.set_device(dev)
-    hbm_peak, tf_peak, tf_sust, peak_src = peaks()
-
-    base = config(1)
-    w = replicate(base, COPIES)
-    t = tensors_torch(w, dev)
-    s = Session(w, t, device=dev, extra_tokens=16)
-    n = base.num_requests
-    steps = []
-    for c in range(COPIES):
-        reqs = copy_requests(w, COPIES, c)
-        ids, q, kn, vn = s.decode_inputs(reqs)   # decode positions == request ids here
-        out, lse = s.new_outputs(len(ids))
-        lens = [w.req_ctx[r] for r in ids]
-        steps.append((B.i32_array(ids), q, kn, vn, out, lse, B.i32_array(lens)))
-    prefix_b, suffix_b, step_bytes = decode_bytes(w, copy_requests(w, COPIES, 0))
+    w, layers, per_layer, setup_s = build_70b_layers(dev, args.layers_70b)
+    n_layers = len(layers)
+    n_dec = len(w.decode_requests())
+    out, lse = layers[0][0].new_outputs(n_dec)
     stream = torch.cuda.current_stream(dev)
+    prefix_b, suffix_b, layer_bytes = decode_bytes(w, w.decode_requests())
+    step_bytes = layer_bytes * n_layers
 
-    def step(i):
-        ids, q, kn, vn, out, lse, lens = steps[i % COPIES]
-        s.ctx.decode(ids, q, kn, vn, out, lse, stream)
-        s.ctx.request_truncate(ids, lens)
+    def step(_i):
+        for s, ida, lna, q, kn, vn in layers:
+            s.ctx.decode(ida, q, kn, vn, out, lse, stream)
+            s.ctx.request_truncate(ida, lna)
 
     def barrier():
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize(dev)
 
-    for i in range(args.warmup):
-        step(i)
-    barrier()
-    props = torch.cuda.get_device_properties(dev)
-    clocks = Clocks(f"GPU-{props.uuid}" if getattr(props, "uuid", None) else str(local_rank))
-    if rank == 0:
-        clocks.start()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for i in range(args.steps):
-        step(args.warmup + i)
-    e1.record(stream)
-    e1.synchronize()
-    ms = e0.elapsed_time(e1)
-    barrier()
-    clk = clocks.stop() if rank == 0 else None
-    ms, bytes_s = job_rate(ms, step_bytes * args.steps, world, dev)
-    launches_per_step = s.ctx.query(B.Q_LAST_LAUNCHES)
-    ms_step = ms / args.steps
-    value = bytes_s / 1e9
-    tokens_s = n * args.steps * world / (ms / 1e3)
-    status = s.ctx.device_status()
 
-    # per-kernel device time (CUDA events on each kernel's stream)
-    s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
-    s.ctx.kernel_times(reset=True)
-    kt_steps = min(args.steps, 400)
-    for i in range(kt_steps):
-        step(i)
-    torch.cuda.synchronize(dev)
-    kt = s.ctx.kernel_times(reset=True)
-    s.ctx.set_option(B.OPT_KERNEL_TIMING, 0)
-    # the unified launch does all of the step's algorithmic HBM work (append,
-    # both levels); the merge that follows only reads the L2-resident partials
-    kbytes = {"dense_tcgen05": step_bytes}
-    share = {k: v[0] for k, v in kt.items() if v[1]}
-    dom = "dense_tcgen05"
-    dom_ms = kt[dom][0] / max(1, kt[dom][1])
-    achieved = kbytes[dom] / (dom_ms / 1e3) / 1e9
-    kernels = {k: {"launches": v[1], "avg_us": round(1e3 * v[0] / v[1], 2) if v[1] else None,
-                   "share": round(v[0] / sum(share.values()), 3) if v[1] else 0.0}
-               for k, v in kt.items() if v[1]}
-
-    # end to end through the public call with host buffers.  A step's inputs
-    # (q, k_new, v_new) sit back to back in one pinned host buffer and its
-    # outputs (out, lse) in another.  tpa_decode takes the pinned host arrays
-    # themselves: its kernels read the inputs and write the outputs over the
-    # CPU-GPU link (NVLink-C2C), so each step moves exactly those bytes across
-    # the link inside the timed region, with no staging copy.  The same step
-    # with copy-engine copies into device buffers and back is timed too.
-    import torch as _t
-
-    def packed(tensors, device):
-        sizes = [x.numel() * x.element_size() for x in tensors]
-        buf = _t.empty(sum(sizes), dtype=_t.uint8, device=device,
-                       pin_memory=device == "cpu")
-        views, off = [], 0
-        for x, n in zip(tensors, sizes):
-            views.append(buf[off:off + n].view(x.dtype).view(x.shape))
-            off += n
-        return buf, views
-
-    host, dev_io = [], []
-    for ids, q, kn, vn, out, lse, lens in steps:
-        hin, hviews = packed((q, kn, vn), "cpu")
-        for hv_, x in zip(hviews, (q, kn, vn)):
-            hv_.copy_(x.cpu())
-        hout, houts = packed((out, lse), "cpu")
-        din, (dq, dkn, dvn) = packed((q, kn, vn), dev)
-        dout, (dou, dls) = packed((out, lse), dev)
-        host.append((hin, hout, hviews, houts))
-        dev_io.append((din, dq, dkn, dvn, dout, dou, dls))
-    h2d = host[0][0].numel()
-    d2h = host[0][1].numel()
-    e2e_steps = args.steps
-
-    def e2e_step(i):
-        ids, _, _, _, _, _, lens = steps[i % COPIES]
-        _, _, (hq, hkn, hvn), (hou, hls) = host[i % COPIES]
-        s.ctx.decode(ids, hq, hkn, hvn, hou, hls, stream)
-        s.ctx.request_truncate(ids, lens)
-
-    def staged_step(i):
-        ids, _, _, _, _, _, lens = steps[i % COPIES]
-        hin, hout, _, _ = host[i % COPIES]
-        din, dq, dkn, dvn, dout, dou, dls = dev_io[i % COPIES]
-        din.copy_(hin, non_blocking=True)
-        s.ctx.decode(ids, dq, dkn, dvn, dou, dls, stream)
-        hout.copy_(dout, non_blocking=True)
-        s.ctx.request_truncate(ids, lens)
-
-    def timed_loop(fn, n):
-        for i in range(args.warmup):
+    def timed_loop(fn, n, clocks=None):
+        for i in range(warmup):
             fn(i)
         barrier()
+        if clocks is not None:
+            clocks.start()
         e0.record(stream)
         for i in range(n):
-            fn(i)
+            fn(warmup + i)
         e1.record(stream)
         e1.synchronize()
-        return e0.elapsed_time(e1)
+        ms = e0.elapsed_time(e1)
+        barrier()
+        clk = clocks.stop() if clocks is not None else None
+        return ms, clk
 
-    ms_e2e, e2e_bytes_s = job_rate(timed_loop(e2e_step, e2e_steps), step_bytes * e2e_steps, world, dev)
-    staged_n = min(e2e_steps, 500)
-    ms_st, st_bytes_s = job_rate(timed_loop(staged_step, staged_n), step_bytes * staged_n, world, dev)
-    e2e = {"value": round(e2e_bytes_s / 1e9, 1), "unit": "GB/s",
-           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-           "ms_per_step": round(ms_e2e / e2e_steps, 4),
-           "io": "pinned host buffers passed to tpa_decode; its kernels read q/k_new/v_new and "
-                 "write out/lse over NVLink-C2C (no staging copy)",
-           "copy_engine": {"value": round(st_bytes_s / 1e9, 1), "unit": "GB/s",
-                           "ms_per_step": round(ms_st / staged_n, 4),
-                           "io": "cudaMemcpyAsync of the packed inputs to device buffers, "
-                                 "tpa_decode on those, cudaMemcpyAsync of the outputs back"}}
+    props = torch.cuda.get_device_properties(dev)
+    clocks = Clocks(f"GPU-{props.uuid}" if getattr(props, "uuid", None) else str(dev.index or 0)) \
+        if rank == 0 else None
+    ms, clk = timed_loop(step, steps, clocks)
+    ms, bytes_s = job_rate(ms, step_bytes * steps, world, dev)
+    launches = sum(s.ctx.query(B.Q_LAST_LAUNCHES) for s, *_ in layers)
+    status = 0
+    for s, *_ in layers:
+        status |= s.ctx.device_status()
+    value = bytes_s / 1e9
+    period_us = 1e3 * ms / (steps * n_layers)
 
-    result = {
+    # per-kernel shares: every launch bracketed by events (two steps, after
+    # one that creates the events)
+    for s, *_ in layers:
+        s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+    step(0)
+    torch.cuda.synchronize(dev)
+    for s, *_ in layers:
+        s.ctx.kernel_times(reset=True)
+    for i in range(2):
+        step(i)
+    torch.cuda.synchronize(dev)
+    kt = {}
+    for s, *_ in layers:
+        for k, v in s.ctx.kernel_times(reset=True).items():
+            a = kt.setdefault(k, [0.0, 0])
+            a[0] += v[0]
+            a[1] += v[1]
+        s.ctx.set_option(B.OPT_KERNEL_TIMING, 0)
+    tot = sum(v[0] for v in kt.values() if v[1]) or 1.0
+    kernels = {k: {"launches": v[1], "bracketed_avg_us": round(1e3 * v[0] / v[1], 1),
+                   "share": round(v[0] / tot, 3)} for k, v in kt.items() if v[1]}
+    dom = "dense_tcgen05"
+    achieved = layer_bytes / (period_us * 1e-6) / 1e9
+    res = {
         "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
+        "steps": steps, "warmup": warmup, "ms_per_step": round(ms / steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) bf16 Q/K/V, random-init; no model weights)",
-        "config": {"workload": "llama3_8b_decode: Hq=32 Hkv=8 d=128 bf16, 4 agents x 4096-token "
-                               "prefixes, 64 decode requests (16/agent), cached suffixes U[256,1024], "
-                               "page 16, contiguous pages",
-                   "l2": f"inputs larger than L2: {COPIES} copies cycled, "
-                         f"{COPIES * step_bytes / 1e9:.2f} GB between reuses",
-                   "bytes_per_step": step_bytes, "prefix_bytes": prefix_b, "suffix_bytes": suffix_b,
-                   "parallelism": f"replicas x{world}"},
+        "config": headline_config(n_layers, world),
+        "ms_per_layer": round(ms / (steps * n_layers), 4),
         "hbm_frac_of_measured": round(value / world / hbm_peak, 4),
         "hbm_frac_of_8tbs": round(value / world / 8000.0, 4),
-        "tokens_per_s": round(tokens_s, 1),
+        "tokens_per_s": round(n_dec * steps * world / (ms / 1e3), 1),
+        "tokens_per_s_note": "decode tokens per second through all layers (one token per request per step)",
         "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1),
                      "peak": hbm_peak, "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
-                     "peak_source": peak_src, "traffic": profiled_traffic(),
-                     "bytes_per_launch": kbytes[dom], "avg_launch_us": round(dom_ms * 1e3, 2)},
+                     "peak_source": peak_src, "traffic": profiled_traffic(PROFILE_70B),
+                     "bytes_per_launch": layer_bytes, "avg_launch_us": round(period_us, 1),
+                     "avg_launch_from": "timed region / unified-kernel launches (back to back)",
+                     "bracketed_avg_us": kernels.get(dom, {}).get("bracketed_avg_us")},
         "kernels": kernels,
-        "e2e": e2e,
-        "gpu_launches": launches_per_step * args.steps,
+        "gpu_launches": launches * steps,
         "clocks": clk,
-        "device_status": status,
+        "resident_gb": round(n_layers * per_layer / 1e9, 1),
+        "setup_s": round(setup_s, 1),
+        "prefix_bytes_per_layer": prefix_b, "suffix_bytes_per_layer": suffix_b,
     }
-    s.ctx.close()
-    del s, t
+
+    if with_e2e:
+        # end to end through the public call with host buffers: each layer's
+        # q, k_new, v_new sit back to back in one pinned host buffer and its
+        # out, lse in another.  tpa_decode takes the pinned host arrays
+        # themselves (its kernels read the inputs and write the outputs over
+        # NVLink-C2C); the same step with copy-engine copies into device
+        # buffers and back is timed too.
+        host, dev_io = [], []
+        for s, ida, lna, q, kn, vn in layers:
+            hin, hviews = _packed((q, kn, vn), "cpu")
+            for hv_, x in zip(hviews, (q, kn, vn)):
+                hv_.copy_(x.cpu())
+            hout, houts = _packed((out, lse), "cpu")
+            din, dviews = _packed((q, kn, vn), dev)
+            dout, douts = _packed((out, lse), dev)
+            host.append((hin, hout, hviews, houts))
+            dev_io.append((din, dout, dviews, douts))
+        h2d = sum(h[0].numel() for h in host)
+        d2h = sum(h[1].numel() for h in host)
+
+        def e2e_step(_i):
+            for (s, ida, lna, *_), (_, _, (hq, hkn, hvn), (hou, hls)) in zip(layers, host):
+                s.ctx.decode(ida, hq, hkn, hvn, hou, hls, stream)
+                s.ctx.request_truncate(ida, lna)
+
+        def staged_step(_i):
+            for (s, ida, lna, *_), (hin, hout, _, _), (din, dout, (dq, dkn, dvn), (dou, dls)) \
+                    in zip(layers, host, dev_io):
+                din.copy_(hin, non_blocking=True)
+                s.ctx.decode(ida, dq, dkn, dvn, dou, dls, stream)
+                hout.copy_(dout, non_blocking=True)
+                s.ctx.request_truncate(ida, lna)
+
+        ms_e, e_bytes_s = job_rate(timed_loop(e2e_step, steps)[0], step_bytes * steps, world, dev)
+        ms_c, c_bytes_s = job_rate(timed_loop(staged_step, steps)[0], step_bytes * steps, world, dev)
+        res["e2e"] = {"value": round(e_bytes_s / 1e9, 1), "unit": "GB/s",
+                      "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                      "ms_per_step": round(ms_e / steps, 4),
+                      "io": "pinned host q/k_new/v_new/out/lse passed to tpa_decode (zero copy)",
+                      "copy_engine": {"value": round(c_bytes_s / 1e9, 1), "unit": "GB/s",
+                                      "ms_per_step": round(ms_c / steps, 4),
+                                      "io": "cudaMemcpyAsync in, tpa_decode, cudaMemcpyAsync out"}}
+        for s, *_ in layers:
+            status |= s.ctx.device_status()
+        del host, dev_io
+    res["device_status"] = status
+    for s, *_ in layers:
+        s.ctx.close()
+    del layers, out, lse
     torch.cuda.empty_cache()
+    return res
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+
+    from paper_2608_25523_gb300.build import build
+
+    build()
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    hbm_peak, tf_peak, tf_sust, peak_src = peaks()
+    result = measure_70b(args, rank, world, dev, hbm_peak, peak_src, args.steps, args.warmup)
     if rank == 0 and world == 1 and not args.no_extras:
+        result["decode_8b"] = bench_decode_8b(args, dev, hbm_peak, peak_src)
         result["prefill"] = bench_prefill(args, dev, tf_peak, peak_src)
-        result["decode_70b"] = bench_70b(args, dev, hbm_peak, peak_src)
         result["mixed"] = bench_mixed(args, dev)
         result["movement"] = bench_movement(args, dev)
         result["redo"] = bench_redo(args, dev)
@@ -384,6 +451,123 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0 and world == 1 and not args.no_cpu:
         result["cpu_baseline"] = cpu_baseline(budget_s=15.0)
     return result
+
+
+def bench_decode_8b(args, dev, hbm_peak, peak_src, steps=2000, warmup=20):
+    """The Llama-3-8B layer decode step: 4 agents x 4096-token prefixes, 64
+    decode requests (16/agent), cached suffixes U[256,1024].  Four copies of
+    the workload are cycled so ~0.93 GB of KV lies between two visits of
+    the same bytes.  Timed over its own `steps` (a 45 us step needs a long
+    region to average out the first step's host latency), with the same e2e
+    variants as the headline."""
+    import torch
+    from paper_2608_25523_gb300 import binding as B
+    from paper_2608_25523_gb300.session import Session
+    from paper_2608_25523_gb300.workloads import config, copy_requests, replicate, tensors_torch
+
+    base = config(1)
+    w = replicate(base, COPIES)
+    t = tensors_torch(w, dev)
+    s = Session(w, t, device=dev, extra_tokens=16)
+    n = base.num_requests
+    steps_io = []
+    for c in range(COPIES):
+        reqs = copy_requests(w, COPIES, c)
+        ids, q, kn, vn = s.decode_inputs(reqs)   # decode positions == request ids here
+        out, lse = s.new_outputs(len(ids))
+        lens = [w.req_ctx[r] for r in ids]
+        steps_io.append((B.i32_array(ids), q, kn, vn, out, lse, B.i32_array(lens)))
+    prefix_b, suffix_b, step_bytes = decode_bytes(w, copy_requests(w, COPIES, 0))
+    stream = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def step(i):
+        ids, q, kn, vn, out, lse, lens = steps_io[i % COPIES]
+        s.ctx.decode(ids, q, kn, vn, out, lse, stream)
+        s.ctx.request_truncate(ids, lens)
+
+    def timed_loop(fn, k):
+        for i in range(warmup):
+            fn(i)
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        for i in range(k):
+            fn(warmup + i)
+        e1.record(stream)
+        e1.synchronize()
+        return e0.elapsed_time(e1)
+
+    ms = timed_loop(step, steps)
+    period_us = 1e3 * ms / steps
+    value = step_bytes / (period_us * 1e-6) / 1e9
+    # a short region at the driver's default size, for comparison
+    ms20 = timed_loop(step, 20)
+
+    s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+    s.ctx.kernel_times(reset=True)
+    for i in range(400):
+        step(i)
+    torch.cuda.synchronize(dev)
+    kt = s.ctx.kernel_times(reset=True)
+    s.ctx.set_option(B.OPT_KERNEL_TIMING, 0)
+    tot = sum(v[0] for v in kt.values() if v[1]) or 1.0
+    kernels = {k: {"launches": v[1], "bracketed_avg_us": round(1e3 * v[0] / v[1], 2),
+                   "share": round(v[0] / tot, 3)} for k, v in kt.items() if v[1]}
+
+    host, dev_io = [], []
+    for ids, q, kn, vn, out, lse, lens in steps_io:
+        hin, hviews = _packed((q, kn, vn), "cpu")
+        for hv_, x in zip(hviews, (q, kn, vn)):
+            hv_.copy_(x.cpu())
+        hout, houts = _packed((out, lse), "cpu")
+        din, dviews = _packed((q, kn, vn), dev)
+        dout, douts = _packed((out, lse), dev)
+        host.append((hin, hout, hviews, houts))
+        dev_io.append((din, dout, dviews, douts))
+
+    def e2e_step(i):
+        ids, _, _, _, _, _, lens = steps_io[i % COPIES]
+        _, _, (hq, hkn, hvn), (hou, hls) = host[i % COPIES]
+        s.ctx.decode(ids, hq, hkn, hvn, hou, hls, stream)
+        s.ctx.request_truncate(ids, lens)
+
+    def staged_step(i):
+        ids, _, _, _, _, _, lens = steps_io[i % COPIES]
+        hin, hout, _, _ = host[i % COPIES]
+        din, dout, (dq, dkn, dvn), (dou, dls) = dev_io[i % COPIES]
+        din.copy_(hin, non_blocking=True)
+        s.ctx.decode(ids, dq, dkn, dvn, dou, dls, stream)
+        hout.copy_(dout, non_blocking=True)
+        s.ctx.request_truncate(ids, lens)
+
+    ms_e = timed_loop(e2e_step, steps)
+    ms_c = timed_loop(staged_step, min(steps, 500))
+    status = s.ctx.device_status()
+    s.ctx.close()
+    del s, t, host, dev_io
+    torch.cuda.empty_cache()
+    dom = "dense_tcgen05"
+    return {"workload": "llama3_8b_decode: Hq32 Hkv8 d128, 4 x 4096-token prefixes, 64 requests, "
+                        "suffixes U[256,1024]",
+            "value": round(value, 1), "unit": "GB/s", "steps": steps, "warmup": warmup,
+            "ms_per_step": round(ms / steps, 5),
+            "hbm_frac_of_measured": round(value / hbm_peak, 4),
+            "hbm_frac_of_8tbs": round(value / 8000.0, 4),
+            "tokens_per_s": round(n / (period_us * 1e-6), 1),
+            "bytes_per_step": step_bytes, "prefix_bytes": prefix_b, "suffix_bytes": suffix_b,
+            "l2": f"{COPIES} copies cycled, {COPIES * step_bytes / 1e9:.2f} GB between reuses",
+            "steps20_ms_per_step": round(ms20 / 20, 5),
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(value, 1),
+                         "peak": hbm_peak, "unit": "GB/s", "frac": round(value / hbm_peak, 4),
+                         "peak_source": peak_src, "traffic": profiled_traffic(PROFILE_8B),
+                         "bytes_per_launch": step_bytes, "avg_launch_us": round(period_us, 2),
+                         "avg_launch_from": "timed region / unified-kernel launches (back to back)",
+                         "bracketed_avg_us": kernels.get(dom, {}).get("bracketed_avg_us")},
+            "kernels": kernels,
+            "e2e": {"value": round(step_bytes * steps / (ms_e / 1e3) / 1e9, 1), "unit": "GB/s",
+                    "ms_per_step": round(ms_e / steps, 4),
+                    "copy_engine_value": round(step_bytes * min(steps, 500) / (ms_c / 1e3) / 1e9, 1)},
+            "device_status": status}
 
 
 def bench_prefill(args, dev, tf_peak, peak_src):
@@ -490,97 +674,6 @@ def bench_sched(args, dev):
                                "cores": 1, "kind": "oracle",
                                "sample": f"the first {n} of {len(rec)} recorded decisions"}
     return out
-
-
-def bench_70b(args, dev, hbm_peak, peak_src):
-    """Llama-3-70B layer decode: 6 agents x 16384-token prefixes, 512
-    requests, suffixes U[512,4096]; 5.3 GB of KV per layer per step.
-
-    The workload is sized to fill most of a 180 GB HBM: L layer pools (one
-    context per layer, all with the same page and request tables, each with
-    its own seeded KV and queries) take about 80 % of 180 GB, capped by the
-    free memory.  A step runs the decode of every layer in turn, as a model's
-    forward pass would, so consecutive decodes never share an L2-resident
-    byte; the numbers are per layer (the step time divided by L)."""
-    import dataclasses
-    import torch
-    from paper_2608_25523_gb300 import binding as B
-    from paper_2608_25523_gb300.session import Session
-    from paper_2608_25523_gb300.workloads import config, tensors_torch
-
-    w = config(4)
-    stream = torch.cuda.current_stream(dev)
-    prefix_b, suffix_b, step_bytes = decode_bytes(w, w.decode_requests())
-    layers = []   # (session, ids array, lens array, q, k_new, v_new)
-    t_setup = time.perf_counter()
-
-    def add_layer(l):
-        wl = w if l == 0 else dataclasses.replace(w, seed=w.seed + 1000 * l)
-        t = tensors_torch(wl, dev)
-        s = Session(wl, t, device=dev, extra_tokens=16, max_tokens=len(w.decode_requests()))
-        ids, q, kn, vn = s.decode_inputs()
-        s.t = None    # the drawn KV now lives in the pool only
-        lens = [w.req_ctx[r] for r in ids]
-        layers.append((s, B.i32_array(ids), B.i32_array(lens), q, kn, vn))
-
-    add_layer(0)
-    torch.cuda.synchronize(dev)
-    s0 = layers[0][0]
-    per_layer = (s0.ctx.k_pool.numel() * 2 * 2 + s0.ctx.workspace.numel()
-                 + 3 * layers[0][3].numel() * 2)
-    free, _ = torch.cuda.mem_get_info(dev)
-    n_layers = max(1, min(args.layers_70b, 1 + int((free - 8e9) // per_layer)))
-    for l in range(1, n_layers):
-        add_layer(l)
-    torch.cuda.synchronize(dev)
-    t_setup = time.perf_counter() - t_setup
-    n_dec = len(w.decode_requests())
-    out, lse = s0.new_outputs(n_dec)
-
-    def step():
-        for s, ida, lna, q, kn, vn in layers:
-            s.ctx.decode(ida, q, kn, vn, out, lse, stream)
-            s.ctx.request_truncate(ida, lna)
-
-    for _ in range(2):
-        step()
-    torch.cuda.synchronize(dev)
-    k = 4
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(k):
-        step()
-    e1.record(stream)
-    e1.synchronize()
-    ms = e0.elapsed_time(e1) / (k * n_layers)
-    for s, *_ in layers:
-        s.ctx.set_option(B.OPT_KERNEL_TIMING, 1)
-    step()
-    kt = {}
-    for s, *_ in layers:
-        for kk, v in s.ctx.kernel_times(reset=True).items():
-            a = kt.setdefault(kk, [0.0, 0])
-            a[0] += v[0]
-            a[1] += v[1]
-    st = 0
-    for s, *_ in layers:
-        st |= s.ctx.device_status()
-        s.ctx.close()
-    resident = n_layers * per_layer
-    del layers, s0, out, lse
-    torch.cuda.empty_cache()
-    gbs = step_bytes / (ms / 1e3) / 1e9
-    return {"workload": "llama3_70b_decode: Hq=64 Hkv=8 d=128, 6 agents x 16384-token prefixes, "
-                        "512 requests, suffixes U[512,4096]; %d layer pools (%.0f GB resident), "
-                        "every step decodes all layers in turn" % (n_layers, resident / 1e9),
-            "layers": n_layers, "resident_gb": round(resident / 1e9, 1),
-            "value": round(gbs, 1), "unit": "GB/s", "ms_per_step": round(ms, 4),
-            "ms_per_step_all_layers": round(ms * n_layers, 3),
-            "hbm_frac_of_measured": round(gbs / hbm_peak, 4), "hbm_frac_of_8tbs": round(gbs / 8000, 4),
-            "tokens_per_s": round(n_dec / (ms / 1e3), 1), "bytes_per_step": step_bytes,
-            "kernels": {kk: {"avg_us": round(1e3 * v[0] / v[1], 1), "launches": v[1]}
-                        for kk, v in kt.items() if v[1]},
-            "setup_s": round(t_setup, 1), "device_status": st}
 
 
 def bench_mixed(args, dev):
@@ -840,56 +933,74 @@ def bench_redo(args, dev):
 
 def bench_coresidency(args, dev):
     """Kernel-level analogue of the paper's Diagnostic 1 (Sec. II, Table 1):
-    under one KV budget, keeping one agent's long prefix resident (Grouped)
-    admits twice the decode batch of keeping two (Alternating).  Budget
-    49152 tokens of one Llama-3-8B layer; prefixes of 16384 tokens; each
-    request holds a 2048-token suffix.  Grouped: agent A resident, 16
-    requests; Alternating: A and B resident, 4 + 4 requests.  Each decode
-    step reads the whole budget either way; throughput follows the batch."""
+    under one KV budget, every further co-resident prefix takes pages that
+    would otherwise hold request suffixes, so the admissible decode batch
+    shrinks.  Budget 49152 tokens of one Llama-3-8B layer; every request
+    holds a 2048-token suffix.  Two prefix lengths:
+
+      16384 tokens  the Grouped / Alternating pair (1 resident prefix
+                    admits 16 requests, 2 admit 8);
+      4096 tokens   1, 2, 3, 4, 6 and 8 resident prefixes.
+
+    The batch is the largest the budget admits, its requests spread
+    round-robin over the resident prefixes.  Each step reads about the
+    whole budget whatever the split, so tokens/s follows the batch.  Two
+    copies of each point's workload are cycled (0.4 GB between reuses)."""
     import torch
     from paper_2608_25523_gb300 import binding as B
     from paper_2608_25523_gb300.session import Session
-    from paper_2608_25523_gb300.workloads import small_case, tensors_torch
+    from paper_2608_25523_gb300.workloads import copy_requests, replicate, small_case, tensors_torch
 
-    lp, ls, budget = 16384, 2048, 49152
-    cases = {"grouped": ([lp], [0] * 16), "alternating": ([lp, lp], [0, 1] * 4)}
-    res = {"workload": f"KV budget {budget} tokens (llama3_8b layer), prefixes {lp}, "
-                       f"suffixes {ls}; decode steps of the admitted batch"}
+    budget, ls = 49152, 2048
+    series = {16384: [1, 2], 4096: [1, 2, 3, 4, 6, 8]}
+    res = {"workload": f"KV budget {budget} tokens (llama3_8b layer), suffixes {ls}; "
+                       "decode steps of the admitted batch", "budget_tokens": budget,
+           "suffix_tokens": ls, "series": {}}
     stream = torch.cuda.current_stream(dev)
-    for name, (plens, agents) in cases.items():
-        n = len(agents)
-        assert sum(plens) + n * ls <= budget
-        w = small_case(7, hq=32, hkv=8, d=128, prefix_len=plens, req_agent=agents,
-                       req_ctx=[ls - 1] * n, req_prefill=[0] * n, req_decode=[1] * n)
-        t = tensors_torch(w, dev)
-        s = Session(w, t, device=dev, extra_tokens=16)
-        ids, q, kn, vn = s.decode_inputs()
-        out, lse = s.new_outputs(n)
-        ida, lna = B.i32_array(ids), B.i32_array([w.req_ctx[r] for r in ids])
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for lp, ks in series.items():
+        pts = []
+        for k in ks:
+            n = (budget - k * lp) // ls
+            agents = [i % k for i in range(n)]
+            base = small_case(7, hq=32, hkv=8, d=128, prefix_len=[lp] * k, req_agent=agents,
+                              req_ctx=[ls - 1] * n, req_prefill=[0] * n, req_decode=[1] * n)
+            assert base.pages_needed() * 16 <= budget
+            w = replicate(base, 2)
+            t = tensors_torch(w, dev)
+            s = Session(w, t, device=dev, extra_tokens=16)
+            io = []
+            for c in range(2):
+                ids, q, kn, vn = s.decode_inputs(copy_requests(w, 2, c))
+                out, lse = s.new_outputs(n)
+                io.append((B.i32_array(ids), B.i32_array([w.req_ctx[r] for r in ids]), q, kn, vn,
+                           out, lse))
 
-        def step():
-            s.ctx.decode(ida, q, kn, vn, out, lse, stream)
-            s.ctx.request_truncate(ida, lna)
-        for _ in range(10):
-            step()
-        torch.cuda.synchronize(dev)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        k = 200
-        e0.record(stream)
-        for _ in range(k):
-            step()
-        e1.record(stream)
-        e1.synchronize()
-        us = e0.elapsed_time(e1) / k * 1e3
-        step_bytes = decode_bytes(w, ids)[2]
-        res[name] = {"resident_prefixes": len(plens), "batch": n, "step_us": round(us, 2),
-                     "tokens_per_s": round(n / (us / 1e6), 1),
-                     "gbs": round(step_bytes / (us / 1e6) / 1e9, 1),
-                     "device_status": s.ctx.device_status()}
-        s.ctx.close()
-        del s, t
-    res["grouped_over_alternating_tokens_per_s"] = round(
-        res["grouped"]["tokens_per_s"] / res["alternating"]["tokens_per_s"], 2)
+            def step(i):
+                ida, lna, q, kn, vn, out, lse = io[i % 2]
+                s.ctx.decode(ida, q, kn, vn, out, lse, stream)
+                s.ctx.request_truncate(ida, lna)
+            for i in range(10):
+                step(i)
+            torch.cuda.synchronize(dev)
+            reps = 400
+            e0.record(stream)
+            for i in range(reps):
+                step(i)
+            e1.record(stream)
+            e1.synchronize()
+            us = e0.elapsed_time(e1) / reps * 1e3
+            step_bytes = decode_bytes(w, copy_requests(w, 2, 0))[2]
+            pts.append({"resident_prefixes": k, "batch": n, "step_us": round(us, 2),
+                        "tokens_per_s": round(n / (us / 1e6), 1),
+                        "gbs": round(step_bytes / (us / 1e6) / 1e9, 1),
+                        "device_status": s.ctx.device_status()})
+            s.ctx.close()
+            del s, t, io
+        res["series"][str(lp)] = pts
+    g, a = res["series"]["16384"]
+    res["grouped_over_alternating_tokens_per_s"] = round(g["tokens_per_s"] / a["tokens_per_s"], 2)
+    torch.cuda.empty_cache()
     return res
 
 
@@ -907,65 +1018,82 @@ def _blas_threads():
 
 
 def cpu_baseline(budget_s=20.0, per_step_s=None, steps=1, warmup=0):
-    """Time the fp64 oracle on this host's cores over a bounded sample of
-    the decode workload.  The sample unit is one (request, kv head): the
-    oracle's decode step for the G query heads of that kv head.  The value
-    scales the step's algorithmic bytes by the fraction of units done."""
-    import oracle
-    from paper_2608_25523_gb300.workloads import config, tensors_numpy
+    """Time the fp64 oracle on this host's cores over a bounded sample of the
+    llama3_70b_decode step (one layer; the per-layer rate is the rate of a
+    step through every layer).  The sample unit is one (request, kv head):
+    the oracle's decode step for the G query heads of that kv head over the
+    request's materialised prefix + suffix + new token.  The units come from
+    16 of the 512 requests, drawn with a fixed seed, with their own suffix
+    lengths; all six prefixes have 16384 tokens, so one drawn prefix stands
+    for each request's.  A unit is credited with the step's algorithmic
+    bytes in proportion to its keys: value = step bytes x (keys of the
+    units done / keys of all 4096 units) / time."""
+    import numpy as np
 
-    w = config(1)
+    import oracle
+    from paper_2608_25523_gb300.workloads import config, small_case, tensors_numpy
+
+    full = config(4)
+    dec = full.decode_requests()
+    step_bytes = decode_bytes(full, dec)[2]
+    hkv, G = full.num_kv_heads, full.group
+    keys_all = sum(full.prefix_len[full.req_agent[r]] + full.req_ctx[r] + 1 for r in dec) * hkv
+    rng = np.random.default_rng(2024)
+    pick = sorted(int(x) for x in rng.choice(len(dec), size=16, replace=False))
+    ctx = [full.req_ctx[dec[i]] for i in pick]
+    lp = full.prefix_len[0]
+    w = small_case(4, hq=full.num_q_heads, hkv=hkv, d=full.head_dim, prefix_len=[lp],
+                   req_agent=[0] * len(pick), req_ctx=ctx, req_prefill=[0] * len(pick),
+                   req_decode=[1] * len(pick))
     t = tensors_numpy(w)
-    dec = w.decode_requests()
-    G, hkv = w.group, w.num_kv_heads
-    units = [(i, g) for i in range(len(dec)) for g in range(hkv)]
-    step_bytes = decode_bytes(w, dec)[2]
+    pk, pv = t.prefix(0, w)
+    units = [(i, g) for i in range(len(pick)) for g in range(hkv)]
 
     def run(us):
+        keys = 0
         for i, g in us:
-            r = dec[i]
-            pk, pv = t.prefix(w.req_agent[r], w)
-            n_cached = w.req_ctx[r] + w.req_prefill[r]
-            sk, sv = t.suffix(r, w, 0, n_cached)
-            nk, nv = t.suffix(r, w, n_cached, n_cached + 1)
+            n_cached = w.req_ctx[i]
+            sk, sv = t.suffix(i, w, 0, n_cached)
+            nk, nv = t.suffix(i, w, n_cached, n_cached + 1)
             oracle.decode_step(t.q_decode[i, g * G:(g + 1) * G], pk[:, g:g + 1], pv[:, g:g + 1],
                                sk[:, g:g + 1], sv[:, g:g + 1], nk[0, g:g + 1], nv[0, g:g + 1])
+            keys += lp + n_cached + 1
+        return keys
 
     t0 = time.perf_counter()
     run(units[:1])
     one = time.perf_counter() - t0
-    total_s, done, pos = 0.0, 0, 0
+    total_s, done_keys, done, pos = 0.0, 0, 0, 0
     if per_step_s is None:
-        # one timed region of about budget_s seconds: units cycled over the step
+        # one timed region of about budget_s seconds, units cycled over the sample
         t_end = time.perf_counter() + budget_s
         t0 = time.perf_counter()
         while done == 0 or time.perf_counter() < t_end:
             k = max(1, min(len(units), int(0.5 / max(one, 1e-6))))
-            run([units[(pos + j) % len(units)] for j in range(k)])
+            done_keys += run([units[(pos + j) % len(units)] for j in range(k)])
             pos += k
             done += k
         total_s = time.perf_counter() - t0
         per = done
     else:
-        per = max(1, min(len(units), int(per_step_s / max(one, 1e-6))))
+        per = max(1, int(per_step_s / max(one, 1e-6)))
         for i in range(warmup + steps):
             sample = [units[(pos + j) % len(units)] for j in range(per)]
             pos += per
             t0 = time.perf_counter()
-            run(sample)
+            kk = run(sample)
             dt = time.perf_counter() - t0
             if i >= warmup:
                 total_s += dt
                 done += per
-    value = step_bytes * (done / len(units)) / total_s / 1e9
+                done_keys += kk
+    frac = done_keys / keys_all
+    value = step_bytes * frac / total_s / 1e9
     return {"value": round(value, 4), "unit": "GB/s", "cores": _blas_threads(), "kind": "oracle",
-            "sample": (f"{done} (request, kv head) units of the llama3_8b_decode step "
-                       f"({len(units)} units per step; {done / len(units):.2f} steps' worth)"
-                       if per_step_s is None else
-                       f"{per} of {len(units)} (request, kv head) units of one llama3_8b_decode "
-                       f"step per timed step, {steps} step(s)")
-                      + "; float64 numpy over per-request materialised KV; value = step bytes x "
-                        "steps' worth done / time",
+            "sample": (f"{done} (request, kv head) units of one llama3_70b_decode layer step "
+                       f"(16 seeded requests x 8 kv heads, cycled; {frac:.3f} layer steps' worth)"
+                       + ("" if per_step_s is None else f", {per} per timed step, {steps} steps")
+                       + "; fp64 numpy over materialised K/V"),
             "seconds": round(total_s, 2)}
 
 
@@ -979,29 +1107,105 @@ def run_reference(args, rank, world):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(1e3 * cb["seconds"] / args.steps, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic",
-            "config": {"workload": "llama3_8b_decode (bounded sample per step, see cpu_baseline)"},
+            "data": "synthetic (seeded N(0,1) bf16-valued Q/K/V)",
+            "config": headline_config(args.layers_70b, world),
             "cpu_baseline": cb,
             "e2e": {"value": cb["value"], "unit": "GB/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
 
+# ------------------------------------------------------------ the line ---
+
+CONTRACT_KEYS = ["metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                 "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config",
+                 "ms_per_layer", "hbm_frac_of_measured", "hbm_frac_of_8tbs", "tokens_per_s",
+                 "roofline", "kernels", "e2e", "gpu_launches", "clocks", "device_status",
+                 "cpu_baseline"]
+
+
+def _csv(xs):
+    return ",".join(str(x) for x in xs)
+
+
+def compact(res):
+    """The printed line: the headline's keys in full and every extra reduced
+    to a few scalars, so the whole line stays short."""
+    out = {k: res[k] for k in CONTRACT_KEYS if k in res}
+    x = res.get("decode_8b")
+    if x:
+        out["decode_8b"] = {"value": x["value"], "unit": "GB/s", "steps": x["steps"],
+                            "ms_per_step": x["ms_per_step"], "frac": x["roofline"]["frac"],
+                            "bracketed_kernel_us": x["roofline"]["bracketed_avg_us"],
+                            "steps20_ms_per_step": x["steps20_ms_per_step"],
+                            "tokens_per_s": x["tokens_per_s"], "e2e_gbs": x["e2e"]["value"],
+                            "traffic": x["roofline"]["traffic"], "device_status": x["device_status"]}
+    x = res.get("prefill")
+    if x:
+        out["prefill"] = {"tflops": x["tflops"], "ms": x["ms"], "tokens_per_s": x["tokens_per_s"],
+                          "kernel_tflops": x["roofline"]["achieved"], "frac": x["roofline"]["frac"],
+                          "peak": x["roofline"]["peak"], "device_status": x["device_status"]}
+    x = res.get("mixed")
+    if x:
+        k = x["kernels_per_step"]
+        out["mixed"] = {"ms_per_step": x["ms_per_step"],
+                        "decode_tokens_per_s": x["decode_tokens_per_s"],
+                        "prefill_kernel_tflops": k.get("prefill_pair_tcgen05", {}).get("tflops"),
+                        "decode_kernel_gbs": k.get("dense_tcgen05", {}).get("gbs"),
+                        "device_status": x["device_status"]}
+    x = res.get("movement")
+    if x:
+        out["movement"] = {"reload_gbs": x["reload"]["B_gbs"], "offload_gbs": x["offload"]["B_gbs"],
+                           "reload_direct_gbs": x["reload_direct"]["B_gbs"],
+                           "offload_direct_gbs": x["offload_direct"]["B_gbs"],
+                           "h2d_copy_gbs": x["h2d_copy"]["B_gbs"],
+                           "mu_over_B_swap_ns": x["mu_over_B_swap_ns_per_token"]["reload"],
+                           "bit_exact": all(r["round_trip_bit_exact"] for r in x["rows"])}
+    x = res.get("redo")
+    if x:
+        out["redo"] = {"tokens": _csv(r["tokens"] for r in x["rows"]),
+                       "decode_kernel_ms": _csv(r["decode_redo_kernel_ms"] for r in x["rows"]),
+                       "prefill_kernel_ms": _csv(r["prefill_rebuild_kernel_ms"] for r in x["rows"]),
+                       "T_decode_us_per_token": x["rows"][-1]["T_decode_us_per_token"],
+                       "device_status": x["device_status"]}
+    x = res.get("coresidency")
+    if x:
+        c = {"budget_tokens": x["budget_tokens"], "suffix_tokens": x["suffix_tokens"]}
+        for lp, pts in x["series"].items():
+            c[f"p{lp}_prefixes"] = _csv(p["resident_prefixes"] for p in pts)
+            c[f"p{lp}_batch"] = _csv(p["batch"] for p in pts)
+            c[f"p{lp}_step_us"] = _csv(p["step_us"] for p in pts)
+            c[f"p{lp}_tokens_per_s"] = _csv(int(p["tokens_per_s"]) for p in pts)
+        c["grouped_over_alternating"] = x["grouped_over_alternating_tokens_per_s"]
+        out["coresidency"] = c
+    x = res.get("sched")
+    if x:
+        out["sched"] = {"tasks": x["tasks"], "decisions": x["decisions"],
+                        "native_decide_us_mean": x["native_decide_us_mean"],
+                        "native_decide_us_max": x["native_decide_us_max"],
+                        "oracle_decide_us": (x.get("cpu_baseline") or {}).get("value"),
+                        "preemptions": x["preemptions"], "prefix_moves_in": x["prefix_moves_in"],
+                        "mean_jct_s": x["mean_jct_s"], "device_status": x["device_status"]}
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--only", choices=["prefill", "decode_70b", "mixed", "movement", "redo",
-                                       "coresidency", "sched"],
-                    help="run just one of the extra workloads (1 GPU) and print its result")
-    ap.add_argument("--layers-70b", type=int, default=26,
+    ap.add_argument("--only", choices=["decode_70b", "decode_8b", "prefill", "mixed", "movement",
+                                       "redo", "coresidency", "sched"],
+                    help="run just one workload (1 GPU) and print its full result")
+    ap.add_argument("--layers-70b", type=int, default=LAYERS_70B,
                     help="layer pools of the 70B decode workload (5.4 GB of KV each; "
                          "26 fill 80 %% of 180 GB), capped by the free memory")
     ap.add_argument("--prefill-stride", type=int, default=1,
                     help="prefill workload: every k-th request only (a small case for profiling)")
+    ap.add_argument("--detail", default=None,
+                    help="also write the full result (every extra in full) to this JSON file")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     rank = int(os.environ.get("RANK", 0))
@@ -1019,8 +1223,11 @@ def main():
         dev = torch.device("cuda", 0)
         torch.cuda.set_device(dev)
         hbm_peak, tf_peak, _, peak_src = peaks()
-        fn = {"prefill": lambda: bench_prefill(args, dev, tf_peak, peak_src),
-              "decode_70b": lambda: bench_70b(args, dev, hbm_peak, peak_src),
+        fn = {"decode_70b": lambda: measure_70b(args, 0, 1, dev, hbm_peak, peak_src, args.steps,
+                                                args.warmup, with_e2e=False),
+              "decode_8b": lambda: bench_decode_8b(args, dev, hbm_peak, peak_src, steps=args.steps,
+                                                   warmup=args.warmup),
+              "prefill": lambda: bench_prefill(args, dev, tf_peak, peak_src),
               "mixed": lambda: bench_mixed(args, dev),
               "movement": lambda: bench_movement(args, dev),
               "redo": lambda: bench_redo(args, dev),
@@ -1035,7 +1242,10 @@ def main():
         dist.init_process_group("nccl")
     res = run_ours(args, rank, world, local_rank)
     if rank == 0:
-        print(json.dumps(res))
+        if args.detail:
+            with open(args.detail, "w") as fh:
+                json.dump(res, fh, indent=1)
+        print(json.dumps(compact(res)))
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()

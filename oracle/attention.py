@@ -25,7 +25,7 @@ definition is used, in float64, over fully materialised per-request K/V:
     o   = sum_j w_j v_j / sum_j w_j
     lse = m + ln(sum_j w_j)             (natural logarithm)
 
-Readings where the paper is silent (each one is listed in the design doc):
+Readings where the paper is silent (the paper prints no attention arithmetic):
   * scale 1/sqrt(d); inputs are post-rotary, synthetic;
   * grouped-query attention: q head h reads kv head h // (Hq / Hkv);
   * decode appends the new token's K/V first, then attends to all

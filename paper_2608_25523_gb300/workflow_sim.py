@@ -25,7 +25,7 @@ from __future__ import annotations
 
 import time
 from dataclasses import dataclass, field
-from typing import List, Optional
+from typing import Callable, List, Optional
 
 import numpy as np
 
@@ -129,9 +129,21 @@ class WorkflowSim:
     def __init__(self, wf: Workflow, ctx: B.Context, *, n_tasks: int, rate: float, seed: int,
                  dims=(8, 2, 64), budget_pages: int, max_tokens: int, max_requests: int,
                  timing: Timing = Timing(), knobs: SchedKnobs = SchedKnobs(),
-                 device: Optional[str] = None, record: Optional[list] = None):
+                 device: Optional[str] = None, record: Optional[list] = None,
+                 on_launch: Optional[Callable] = None):
         self.wf, self.ctx, self.tm, self.kn = wf, ctx, timing, knobs
         self.record = record   # if a list: every decision's (params, snapshot, decision)
+        # Called after every prefill chunk as on_launch(self, "prefill", (lib_id, offset, c))
+        # and after every decode step as on_launch(self, "decode", ids), with the
+        # launches still in flight.  kv_log[lib_id] lists what the request's suffix
+        # holds, in order: ("pf", c) = rows 0..c-1 of k_pf / v_pf (one prefill
+        # chunk), ("dec", j) = row j of k_dec / v_dec (one decode token); events
+        # lists ("reload", agent), ("preempt", lib_id) and ("rebuild", lib_id,
+        # tokens) in the order they happened.
+        self.on_launch = on_launch
+        self.kv_log = {}
+        self.lib_agent = {}     # lib_id -> agent of the request it holds
+        self.events = []
         self.hq, self.hkv, self.d = dims
         self.budget_tokens = budget_pages * PAGE
         self.max_tokens = max_tokens
@@ -181,6 +193,7 @@ class WorkflowSim:
         else:
             hk, hv = self.host_kv.get(a, (1, 1))
             self.ctx.prefix_reload(a, hk, hv)
+            self.events.append(("reload", a))
         self.agent_state[a] = "resident"
         self.res.prefix_in += 1
 
@@ -199,6 +212,9 @@ class WorkflowSim:
                                        self.o_pf, self.l_pf)
             else:
                 self.ctx.prefill_chunk([lib_id], [c], 1, 1, 1, 1, 1)
+            self.kv_log.setdefault(lib_id, []).append(("pf", c))
+            if self.on_launch is not None:
+                self.on_launch(self, "prefill", (lib_id, done, c))
             done += c
         self.res.prefill_tokens += ntok
 
@@ -209,6 +225,10 @@ class WorkflowSim:
                             self.o_dec[:n], self.l_dec[:n])
         else:
             self.ctx.decode(ids, 1, 1, 1, 1, 1)
+        for j, i in enumerate(ids):
+            self.kv_log.setdefault(i, []).append(("dec", j))
+        if self.on_launch is not None:
+            self.on_launch(self, "decode", list(ids))
         self.res.decode_tokens += len(ids)
 
     # ------------------------------------------------------------ state
@@ -269,6 +289,7 @@ class WorkflowSim:
             # completions (committed before the next decision)
             for r in [r for r in running if r.generated >= wf.output_tokens[r.stage]]:
                 self.ctx.request_close(r.lib_id)
+                self.kv_log.pop(r.lib_id, None)
                 self.free_ids.append(r.lib_id)
                 reqs.remove(r)
                 tk = tasks[r.task]
@@ -329,6 +350,8 @@ class WorkflowSim:
         for i, r in enumerate(reqs):
             if r.running and i not in keep:
                 self.ctx.request_close(r.lib_id)
+                self.kv_log.pop(r.lib_id, None)
+                self.events.append(("preempt", r.lib_id))
                 self.free_ids.append(r.lib_id)
                 r.running, r.lib_id, r.credit = False, -1, 0.0
                 r.redo = r.generated          # y_r: rebuilt on re-admission
@@ -349,7 +372,11 @@ class WorkflowSim:
             r = reqs[i]
             r.lib_id = self.free_ids.pop()
             self.ctx.request_open(r.lib_id, wf.stage_agent[r.stage])
+            self.kv_log[r.lib_id] = []
+            self.lib_agent[r.lib_id] = wf.stage_agent[r.stage]
             ntok = self.wf.input_tokens[r.stage] + r.redo
+            if r.redo:
+                self.events.append(("rebuild", r.lib_id, ntok))
             self._prefill(r.lib_id, ntok)
             r.generated, r.redo = r.redo, 0
             r.running, r.credit = True, lam

@@ -2,22 +2,28 @@
 
 Inputs are drawn on the device by the seeded generator (workloads.tensors_torch);
 only the slices the oracle needs are copied to the host, in float64.  Rows
-are checked against the fp64 oracle one by one:
+are checked against the fp64 oracle:
 
   * llama3_8b_decode: the bench's 4-copy context, the steps of copies 0
     and 3, every row;
-  * llama3_70b_decode: one step, a seeded sample of 64 of the 512 requests
-    (every head);
+  * llama3_70b_decode: one step, all 512 requests (every head; so every
+    dense tile and every split-KV item of the launch);
   * chunked_prefill: every 512-token chunk round of the 256 new requests,
-    with a seeded sample of rows per round (first and last row of a chunk
-    included);
+    the first, the last and one seeded row of every chunk;
   * mixed: reload of 2 evicted prefixes on a side stream (bit-exact), the
-    8 prefill chunks (sampled rows) and all 256 Zipf decode requests in one
-    step.
+    8 prefill chunks (32 rows each, first and last included) and all 256
+    Zipf decode requests in one step;
+  * the co-residency points of the bench (one 16384-token prefix with 16
+    requests of 2048 tokens, two with 8, eight 4096-token prefixes with one
+    request each), every row of both copies' steps.
 
 A causal prefill row at suffix position p sees the whole prefix and suffix
 positions 0..p, which is the oracle's decode step with suffix[0:p] cached
-and suffix[p] as the step's own token; sampled rows are checked that way.
+and suffix[p] as the step's own token.  For the large sets of rows the
+oracle's answer is assembled from two oracle.attend calls, one over the
+agent's prefix (all of that agent's rows at once) and one over the
+request's suffix rows, joined by oracle.lse_merge: the exact merge the
+oracle's pins check against single-pass attention (tests/test_oracle_pins.py).
 """
 import numpy as np
 import pytest
@@ -27,7 +33,8 @@ import oracle
 from paper_2608_25523_gb300 import binding as B
 from paper_2608_25523_gb300.build import build
 from paper_2608_25523_gb300.session import Session
-from paper_2608_25523_gb300.workloads import config, copy_requests, replicate, tensors_torch
+from paper_2608_25523_gb300.workloads import (config, copy_requests, replicate, small_case,
+                                               tensors_torch)
 
 from _util import compare
 
@@ -67,12 +74,47 @@ def _decode_ref(w, t, r, q_row):
     return oracle.decode_step(_h(q_row), pk, pv, _h(sk), _h(sv), _h(nk[0]), _h(nv[0]))
 
 
-def _prefill_row_ref(w, t, r, p, q_row):
-    """Oracle output of request r's prefill row at suffix position p."""
-    pk, pv = _prefix_host(w, t, w.req_agent[r])
-    sk, sv = t.suffix(r, w, 0, p)
-    nk, nv = t.suffix(r, w, p, p + 1)
-    return oracle.decode_step(_h(q_row), pk, pv, _h(sk), _h(sv), _h(nk[0]), _h(nv[0]))
+def _refs_by_parts(w, t, items):
+    """fp64 oracle output of query rows.  items: (request r, keys k, q_row
+    [Hq, d] float64), a row that sees the whole prefix of r's agent and r's
+    suffix rows 0..k-1.  Computed as oracle.attend over the prefix (all rows
+    of one agent and kv head in one call), oracle.attend over the suffix
+    rows, and oracle.lse_merge of the two.  Returns o [n, Hq, d], lse [n, Hq]."""
+    hq, hkv, d, G = w.num_q_heads, w.num_kv_heads, w.head_dim, w.group
+    n = len(items)
+    Q = np.stack([q for _, _, q in items])
+    o_pre = np.zeros((n, hq, d))
+    l_pre = np.zeros((n, hq))
+    by_agent, by_req = {}, {}
+    for i, (r, _, _) in enumerate(items):
+        by_agent.setdefault(w.req_agent[r], []).append(i)
+        by_req.setdefault(r, []).append(i)
+    for a, idx in by_agent.items():
+        if w.prefix_len[a] == 0:
+            continue
+        pk, pv = t.prefix(a, w)
+        for g in range(hkv):
+            rows = Q[idx][:, g * G:(g + 1) * G].reshape(-1, d)
+            o, l = oracle.attend(rows, _h(pk[:, g]), _h(pv[:, g]))
+            o_pre[idx, g * G:(g + 1) * G] = o.reshape(len(idx), G, d)
+            l_pre[idx, g * G:(g + 1) * G] = l.reshape(len(idx), G)
+    O = np.empty((n, hq, d))
+    L = np.empty((n, hq))
+    for r, idx in by_req.items():
+        sk, sv = t.suffix(r, w, 0, max(items[i][1] for i in idx))
+        SK, SV = _h(sk), _h(sv)
+        for i in idx:
+            k = items[i][1]
+            o_s = np.empty((hq, d))
+            l_s = np.empty(hq)
+            for g in range(hkv):
+                o_s[g * G:(g + 1) * G], l_s[g * G:(g + 1) * G] = oracle.attend(
+                    Q[i, g * G:(g + 1) * G], SK[:k, g], SV[:k, g])
+            if w.prefix_len[w.req_agent[r]] == 0:
+                O[i], L[i] = o_s, l_s
+            else:
+                O[i], L[i] = oracle.lse_merge([(o_pre[i], l_pre[i]), (o_s, l_s)])
+    return O, L
 
 
 def _check_rows(out, lse, refs, what):
@@ -101,24 +143,24 @@ def test_llama3_8b_decode_bench_context():
     s.ctx.close()
 
 
-def test_llama3_70b_decode_sampled():
+def test_llama3_70b_decode_all_requests():
     w = config(4)
     t = tensors_torch(w, "cuda")
-    s = Session(w, t, extra_tokens=16)
+    s = Session(w, t, extra_tokens=16, max_tokens=len(w.decode_requests()))
     ids, q, kn, vn = s.decode_inputs()
     out, lse = s.new_outputs(len(ids))
     s.decode(ids, q, kn, vn, out, lse)
     torch.cuda.synchronize()
     assert s.ctx.device_status() == 0
-    rng = np.random.default_rng(404)
-    pick = sorted(rng.choice(len(ids), size=64, replace=False).tolist())
-    refs = [_decode_ref(w, t, ids[k], q[k]) for k in pick]
-    idx = torch.tensor(pick, device="cuda")
-    _check_rows(out[idx], lse[idx], refs, "llama3_70b_decode sample")
+    assert s.ctx.query(B.Q_LAST_DENSE_ITEMS) > 0 and s.ctx.query(B.Q_LAST_SUFFIX_ITEMS) > 0
+    qh = _h(q)
+    items = [(r, w.req_ctx[r] + 1, qh[k]) for k, r in enumerate(ids)]
+    o_ref, l_ref = _refs_by_parts(w, t, items)
+    compare(out, lse, o_ref, l_ref, "llama3_70b_decode, all 512 requests")
     s.ctx.close()
 
 
-def test_chunked_prefill_all_rounds_sampled():
+def test_chunked_prefill_all_rounds_every_chunk():
     w = config(2)
     t = tensors_torch(w, "cuda")
     s = Session(w, t, extra_tokens=0)
@@ -130,15 +172,15 @@ def test_chunked_prefill_all_rounds_sampled():
         torch.cuda.synchronize()
         assert s.ctx.device_status() == 0
         starts = np.cumsum([0] + lens[:-1])
-        rows, refs = [], []
-        for ci in sorted(rng.choice(len(chunks), size=min(16, len(chunks)), replace=False).tolist()):
-            r, off, c = chunks[ci]
+        rows, items = [], []
+        for ci, (r, off, c) in enumerate(chunks):
             for i in sorted({0, c - 1, int(rng.integers(0, c))}):
                 row = int(starts[ci]) + i
                 rows.append(row)
-                refs.append(_prefill_row_ref(w, t, r, off + i, q[row]))
+                items.append((r, off + i + 1, _h(q[row])))
+        o_ref, l_ref = _refs_by_parts(w, t, items)
         idx = torch.tensor(rows, device="cuda")
-        _check_rows(out[idx], lse[idx], refs, f"chunked_prefill round {rnd}")
+        compare(out[idx], lse[idx], o_ref, l_ref, f"chunked_prefill round {rnd}, {len(rows)} rows")
     s.ctx.close()
 
 
@@ -172,11 +214,40 @@ def test_mixed_step():
     refs = [_decode_ref(w, t, r, dq[k]) for k, r in enumerate(dids)]
     _check_rows(dout, dlse, refs, "mixed decode")
     starts = np.cumsum([0] + plens[:-1])
-    rows, prefs = [], []
+    rows, items = [], []
     for ci, (r, off, c) in enumerate(chunks):
-        for i in sorted({0, c - 1, int(rng.integers(0, c))}):
-            rows.append(int(starts[ci]) + i)
-            prefs.append(_prefill_row_ref(w, t, r, off + i, pq[int(starts[ci]) + i]))
+        pick = {0, c - 1} | {int(x) for x in rng.choice(c, size=min(c, 30), replace=False)}
+        for i in sorted(pick):
+            row = int(starts[ci]) + i
+            rows.append(row)
+            items.append((r, off + i + 1, _h(pq[row])))
+    o_ref, l_ref = _refs_by_parts(w, t, items)
     idx = torch.tensor(rows, device="cuda")
-    _check_rows(pout[idx], plse[idx], prefs, "mixed prefill sample")
+    compare(pout[idx], plse[idx], o_ref, l_ref, f"mixed prefill, {len(rows)} rows")
+    s.ctx.close()
+
+
+@pytest.mark.parametrize("lp,k", [(16384, 1), (16384, 2), (4096, 8)],
+                         ids=["grouped_16384x1", "alternating_16384x2", "prefixes_4096x8"])
+def test_coresidency_points(lp, k):
+    """The co-residency bench's shapes: a 49152-token budget, 2048-token
+    suffixes, k resident prefixes of lp tokens and the batch the budget
+    admits, two copies cycled as the bench does."""
+    budget, ls = 49152, 2048
+    n = (budget - k * lp) // ls
+    base = small_case(7, hq=32, hkv=8, d=128, prefix_len=[lp] * k, req_agent=[i % k for i in range(n)],
+                      req_ctx=[ls - 1] * n, req_prefill=[0] * n, req_decode=[1] * n)
+    w = replicate(base, 2)
+    t = tensors_torch(w, "cuda")
+    s = Session(w, t, extra_tokens=16)
+    for c in (0, 1):
+        ids, q, kn, vn = s.decode_inputs(copy_requests(w, 2, c))
+        out, lse = s.new_outputs(len(ids))
+        s.decode(ids, q, kn, vn, out, lse)
+        torch.cuda.synchronize()
+        assert s.ctx.device_status() == 0
+        qh = _h(q)
+        items = [(r, w.req_ctx[r] + 1, qh[j]) for j, r in enumerate(ids)]
+        o_ref, l_ref = _refs_by_parts(w, t, items)
+        compare(out, lse, o_ref, l_ref, f"coresidency {k} x {lp}, batch {n}, copy {c}")
     s.ctx.close()
