@@ -220,7 +220,11 @@ TPA_API int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void*
  *   outputs [slots][d] followed by their fp32 LSEs, so it holds
  *   slots = (16 MiB - 256) / (4 (d + 1)) partials (32510 at d = 128).  Its
  *   address is looked up once per device (with that device current) and
- *   cached; the call allocates no device or pinned memory.
+ *   cached; the call allocates no device or pinned memory.  Under lazy
+ *   module loading (CUDA's default) only a context that runs this entry
+ *   point loads the array; with CUDA_MODULE_LOADING=EAGER every context that
+ *   loads the library holds it.  The cached address is the primary
+ *   context's: after cudaDeviceReset do not call this entry point again.
  *   Nothing in the array has to start at zero: every partial a call reads
  *   is written earlier in the same call.
  *   All calls of this entry point on one device share the array: calls

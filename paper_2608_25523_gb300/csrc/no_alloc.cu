@@ -1,7 +1,10 @@
 // Fixed device scratch for tpa_decode_static_scratch: the split-KV partial
 // results of one decode call live in a file-scope device array of this
-// translation unit (its own module, so the array is only loaded by callers
-// of that entry point) instead of the workspace the caller allocated.
+// translation unit instead of the workspace the caller allocated.  Under
+// lazy module loading (CUDA's default) only a context that runs this entry
+// point loads the array; with CUDA_MODULE_LOADING=EAGER every context that
+// loads the library holds it.  The address is cached per device: it is the
+// primary context's, valid until that context is destroyed (cudaDeviceReset).
 #include <cuda_runtime.h>
 
 #include <mutex>

@@ -3,7 +3,8 @@
 The variant keeps the split partials of a decode step in the library's
 static device array instead of the context workspace; everything else is
 tpa_decode, so two decode steps in a row must give bit-identical outputs
-and leave bit-identical KV pages.  A step needing more partials than the
+and leave bit-identical KV pages, and the context workspace must keep its
+partials untouched.  A step needing more partials than the
 array holds is refused with a CAPACITY error that names the limit, and
 changes nothing.  Collected last, so it runs both alone and after every
 other GPU test in the same process.
@@ -86,6 +87,39 @@ def test_two_steps_bit_identical_to_decode(mode):
         assert torch.equal(_bits(kr), _bits(kv)) and torch.equal(_bits(vr), _bits(vv))
     ref.ctx.close()
     var.ctx.close()
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
+def test_workspace_partials_untouched(mode):
+    """The partials really live in the static array: after a tpa_decode
+    step, the same step with other inputs through tpa_decode_static_scratch
+    changes only the plan upload in the context workspace, while through
+    tpa_decode it rewrites the workspace's partials (far more bytes)."""
+    w = _workload(71 + mode)
+    s = Session(w, to_device(tensors_numpy(w), "cuda"))
+    s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+    ids = list(range(w.num_requests))
+    lens = [s.ctx.query(B.Q_SUFFIX_LEN, r) for r in ids]
+    out, lse = s.new_outputs(len(ids))
+    ws = s.ctx.workspace
+
+    def changed_by(fn, seed):
+        q, kn, vn = _step_inputs(w, len(ids), seed)
+        before = ws.clone()
+        fn(ids, q, kn, vn, out, lse)
+        torch.cuda.synchronize()
+        s.ctx.request_truncate(ids, lens)
+        return int((ws != before).sum())
+
+    changed_by(s.ctx.decode, 1)
+    static = changed_by(s.ctx.decode_static_scratch, 2)
+    regular = changed_by(s.ctx.decode, 3)
+    assert s.ctx.device_status() == 0
+    # the step's partials: at least one per (token, q head), (d + 1) fp32 each
+    partial_bytes = len(ids) * w.num_q_heads * (w.head_dim + 1) * 4
+    assert static < partial_bytes // 4, (static, partial_bytes)
+    assert regular > partial_bytes // 2, (regular, partial_bytes)
+    s.ctx.close()
 
 
 def test_oversize_step_refused():
