@@ -289,6 +289,11 @@ enum {
                                    staging area, and scatters / gathers the pages on the device;
                                    0 runs the page kernel on the mapped host arrays directly (it
                                    holds its SMs for the whole link-bound transfer) */
+  TPA_OPT_TEST_BAD_SLOT = 9     /* test hook, 1: the next decode's plan gives its first token
+                                   partial slots past the end of the partial buffer.  Every
+                                   kernel checks partial slots: that token's partials are neither
+                                   written nor read, its outputs are left unwritten and the
+                                   device status gets bit 16; later steps are unaffected */
 };
 TPA_API int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value);
 
@@ -307,7 +312,8 @@ TPA_API int tpa_kernel_times(tpa_ctx* ctx, int32_t n, double* total_ms, int64_t*
  * *status = 0 when no kernel reported a problem; otherwise a bit set:
  * 1 a dense-kernel wait timed out, 2 a suffix-kernel wait timed out,
  * 4 a page id outside the pool was met (the access was redirected to page
- * 0), 8 a kernel gave up waiting for its plan upload (it did no work).
+ * 0), 8 a kernel gave up waiting for its plan upload (it did no work),
+ * 16 a partial slot outside the partial buffer was met (not written or read).
  * Returns TIMEOUT if bit 1, 2 or 8 is set, CUDA on a CUDA error. */
 TPA_API int tpa_device_status(tpa_ctx* ctx, void* stream, uint32_t* status);
 

@@ -39,6 +39,7 @@ OPT_TEST_PLAN_WAIT = 5
 OPT_PREFILL_TILE_ROWS = 6
 OPT_TEST_BAD_PAGE = 7
 OPT_MOVEMENT_STAGED = 8
+OPT_TEST_BAD_SLOT = 9
 # kernel kinds of tpa_kernel_times
 KERNEL_NAMES = ["kv_append", "dense_tcgen05", "split_kv", "lse_merge", "page_copy",
                 "prefill_pair_tcgen05"]

@@ -168,6 +168,7 @@ struct tpa_ctx {
   bool staged_movement = true;  // TPA_OPT_MOVEMENT_STAGED  // query rows per prefill work item: 256 (tile pairs) or 128
   int test_plan_wait = 0;  // test hook: the next cascade decode waits for a flag never written
   int test_bad_page = 0;   // test hook: the next decode's first prefix page id is out of the pool
+  int test_bad_slot = 0;   // test hook: the next decode's first token's partial slots are out of range
   int prefix_splits = 0;
   int suffix_split_keys = 0;
   int64_t last_dense = 0, last_suffix = 0, last_launches = 0;
@@ -1023,6 +1024,7 @@ static DenseParams dense_params(tpa_ctx* ctx, const Slot* sl, const PlanLayout& 
   dp.lse = lse;
   dp.part_o = ctx->part_o;
   dp.part_lse = ctx->part_lse;
+  dp.part_slots = ctx->part_slots;
   dp.items = dev_ptr<DenseItem>(sl, lay.off_dense);
   dp.toks = dev_ptr<DenseTok>(sl, lay.off_dense_tok);
   dp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
@@ -1190,6 +1192,12 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
     slots += static_cast<int64_t>(hq) * ns;
   }
   if (slots > ctx->part_slots) return fail(TPA_ERR_CAPACITY, "partial slots exhausted");
+  if (ctx->test_bad_slot && n > 0) {
+    // every kernel checks partial slots against the buffer: nothing of this
+    // token's partials is written or read
+    slot_base[0] = static_cast<int32_t>(std::min<int64_t>(ctx->part_slots, INT32_MAX));
+    ctx->test_bad_slot = 0;
+  }
 
   // plan sizes (suffix page counts after this step's append)
   PlanSizes sz;
@@ -1350,6 +1358,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       sp.q = static_cast<const __nv_bfloat16*>(q);
       sp.part_o = ctx->part_o;
       sp.part_lse = ctx->part_lse;
+      sp.part_slots = ctx->part_slots;
       sp.items = dev_ptr<SuffixItem>(sl, lay.off_suffix);
       sp.pages = dev_ptr<int32_t>(sl, lay.off_pages);
       sp.queue = reinterpret_cast<uint32_t*>(sl->dev + offsetof(PlanHeader, queue));
@@ -1366,6 +1375,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
       {
         KernelTimer kt(ctx, K_MERGE, s);
         CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
+                              ctx->part_slots, ctx->status,
                               static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, ctx->num_sms,
                               true, s));
       }
@@ -1403,6 +1413,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
         // a programmatic dependent: resident before the main kernel ends
         KernelTimer kt(ctx, K_MERGE, s);
         CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
+                              ctx->part_slots, ctx->status,
                               static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, ctx->num_sms,
                               true, s));
       }
@@ -1717,6 +1728,9 @@ int tpa_set_option(tpa_ctx* ctx, int32_t option, int64_t value) {
       return TPA_OK;
     case TPA_OPT_TEST_BAD_PAGE:
       ctx->test_bad_page = value ? 1 : 0;
+      return TPA_OK;
+    case TPA_OPT_TEST_BAD_SLOT:
+      ctx->test_bad_slot = value ? 1 : 0;
       return TPA_OK;
     case TPA_OPT_MOVEMENT_STAGED:
       ctx->staged_movement = value != 0;

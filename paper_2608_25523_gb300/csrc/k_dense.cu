@@ -123,7 +123,7 @@ __device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) 
   SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, nullptr, p.n_sitems,
               p.stoks, p.full_prefix, p.tail_order, p.n_stok, p.n_full, p.split_keys, p.pages,
               p.squeue, p.status, p.num_pages, p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new,
-              p.k_pool, p.v_pool};
+              p.k_pool, p.v_pool, p.part_slots};
   split_warp_loop<D, G, kSplitStages>(a, ring, bars, abort_flag, lane);
 }
 
@@ -511,6 +511,9 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
       const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
       const float lse = l_tot > 0.f ? (m_run + __log2f(l_tot)) * kLn2 : -INFINITY;
       const int64_t slot = dt.slot_base + static_cast<int64_t>(head) * dt.n_slots + item.split;
+      // a partial slot outside the partial buffer is not written (status bit)
+      const bool slot_ok = item.out_mode != 0 || (slot >= 0 && slot < p.part_slots);
+      if (ok && row_valid && !slot_ok) atomicOr(p.status, kStatusBadSlot);
       if (ok) {
         tc_fence_after();
 #pragma unroll 1
@@ -519,7 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           const int col = half * (D / 2) + 32 * c;
           tmem_ld32(tmem + lane_base + C::kColO + col, o);
           tmem_wait_ld();
-          if (row_valid) {
+          if (row_valid && slot_ok) {
             if (item.out_mode == 0) {
               float4* dst = reinterpret_cast<float4*>(p.part_o + slot * D + col);
 #pragma unroll
@@ -542,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           }
         }
         tc_fence_before();
-        if (row_valid && half == 0) {
+        if (row_valid && slot_ok && half == 0) {
           if (item.out_mode == 0) p.part_lse[slot] = lse;
           else p.lse[static_cast<int64_t>(dt.q_row) * p.hq + head] = lse;
         }

@@ -25,8 +25,8 @@ constexpr int kMergeThreads = 128;
 template <int D>
 __global__ void __launch_bounds__(kMergeThreads)
     merge_kernel(const MergeTok* __restrict__ toks, int n_tok, const float* __restrict__ part_o,
-                 const float* __restrict__ part_lse, __nv_bfloat16* __restrict__ out,
-                 float* __restrict__ lse_out, int hq) {
+                 const float* __restrict__ part_lse, int64_t part_slots, uint32_t* status,
+                 __nv_bfloat16* __restrict__ out, float* __restrict__ lse_out, int hq) {
   pdl_trigger();  // the next step's main kernel may become resident now
   pdl_wait();     // no-op unless launched as a dependent
   constexpr int LPI = D / 4;     // lanes per (token, head)
@@ -41,6 +41,11 @@ __global__ void __launch_bounds__(kMergeThreads)
     const MergeTok m = toks[t];
     const int64_t base = m.slot_base + static_cast<int64_t>(h) * m.n_slots;
     const int col = 4 * (lane % LPI);
+    if (base < 0 || m.n_slots < 0 || base + m.n_slots > part_slots) {
+      // partial slots outside the partial buffer: not read (status bit)
+      if (lane % LPI == 0) atomicOr(status, kStatusBadSlot);
+      continue;
+    }
     float acc[4], mx, tot;
     merge_partials<1, 8>(part_lse + base, part_o + base * D + col, m.n_slots, D, acc, mx, tot);
     const float inv = tot > 0.f ? 1.f / tot : 0.f;
@@ -56,8 +61,9 @@ __global__ void __launch_bounds__(kMergeThreads)
 
 template <int D>
 cudaError_t launch_merge_t(const MergeTok* toks, int n_tok, const float* part_o,
-                           const float* part_lse, __nv_bfloat16* out, float* lse, int hq,
-                           int num_sms, bool dependent, cudaStream_t stream) {
+                           const float* part_lse, int64_t part_slots, uint32_t* status,
+                           __nv_bfloat16* out, float* lse, int hq, int num_sms, bool dependent,
+                           cudaStream_t stream) {
   constexpr int IPB = (kMergeThreads / 32) * (32 / (D / 4));  // pairs per block and pass
   const int64_t pairs = static_cast<int64_t>(n_tok) * hq;
   int64_t blocks = (pairs + IPB - 1) / IPB;
@@ -73,21 +79,23 @@ cudaError_t launch_merge_t(const MergeTok* toks, int n_tok, const float* part_o,
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = dependent ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, merge_kernel<D>, toks, n_tok, part_o, part_lse, out, lse, hq);
+  return cudaLaunchKernelEx(&cfg, merge_kernel<D>, toks, n_tok, part_o, part_lse, part_slots, status,
+                            out, lse, hq);
 }
 
 }  // namespace
 
 cudaError_t launch_merge(const MergeTok* toks, int n_tok, const float* part_o,
-                         const float* part_lse, __nv_bfloat16* out, float* lse, int hq, int d,
-                         int num_sms, bool dependent, cudaStream_t stream) {
+                         const float* part_lse, int64_t part_slots, uint32_t* status,
+                         __nv_bfloat16* out, float* lse, int hq, int d, int num_sms,
+                         bool dependent, cudaStream_t stream) {
   if (n_tok <= 0) return cudaSuccess;
   if (d == 128)
-    return launch_merge_t<128>(toks, n_tok, part_o, part_lse, out, lse, hq, num_sms, dependent,
-                               stream);
+    return launch_merge_t<128>(toks, n_tok, part_o, part_lse, part_slots, status, out, lse, hq,
+                               num_sms, dependent, stream);
   if (d == 64)
-    return launch_merge_t<64>(toks, n_tok, part_o, part_lse, out, lse, hq, num_sms, dependent,
-                              stream);
+    return launch_merge_t<64>(toks, n_tok, part_o, part_lse, part_slots, status, out, lse, hq,
+                              num_sms, dependent, stream);
   return cudaErrorInvalidValue;
 }
 

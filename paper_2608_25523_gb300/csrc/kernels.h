@@ -42,6 +42,7 @@ struct DenseParams {
   float* lse;
   float* part_o;
   float* part_lse;
+  int64_t part_slots;  // entries of part_lse (part_o: part_slots x d); other slots are refused
   const DenseItem* items;
   const DenseTok* toks;
   const int32_t* pages;
@@ -91,6 +92,7 @@ struct SuffixParams {
   const __nv_bfloat16* q;
   float* part_o;
   float* part_lse;
+  int64_t part_slots;  // entries of part_lse (part_o: part_slots x d); other slots are refused
   const SuffixItem* items;
   const int32_t* pages;
   uint32_t* queue;     // zeroed work counter
@@ -115,8 +117,9 @@ cudaError_t launch_suffix(const SuffixParams& p, int num_sms, int head_dim, int 
 // before it on the stream (which triggers early): its CTAs become resident
 // while that kernel still runs and start merging the moment it completes.
 cudaError_t launch_merge(const MergeTok* toks, int n_tok, const float* part_o,
-                         const float* part_lse, __nv_bfloat16* out, float* lse, int hq, int d,
-                         int num_sms, bool dependent, cudaStream_t stream);
+                         const float* part_lse, int64_t part_slots, uint32_t* status,
+                         __nv_bfloat16* out, float* lse, int hq, int d, int num_sms,
+                         bool dependent, cudaStream_t stream);
 
 // Raise dynamic shared-memory limits of the kernels (once per device).
 cudaError_t init_kernels();

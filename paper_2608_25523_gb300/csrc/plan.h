@@ -14,6 +14,7 @@ constexpr uint32_t kStatusDenseTimeout = 1u;
 constexpr uint32_t kStatusSuffixTimeout = 2u;
 constexpr uint32_t kStatusBadPage = 4u;
 constexpr uint32_t kStatusPlanTimeout = 8u;  // a plan upload never arrived
+constexpr uint32_t kStatusBadSlot = 16u;     // a partial slot outside the partial buffer (skipped)
 
 // A run of a KV write within one page: source rows src .. src + n - 1 of
 // the K/V arrays go to slots slot .. slot + n - 1 of page `page` (n <= 16).

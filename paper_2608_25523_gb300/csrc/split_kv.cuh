@@ -54,6 +54,7 @@ struct SplitArgs {
   const __nv_bfloat16* v_new;
   __nv_bfloat16* k_pool;
   __nv_bfloat16* v_pool;
+  int64_t part_slots;  // entries of part_lse; a slot outside [0, part_slots) is not written
 };
 
 template <int D, int S>
@@ -311,9 +312,12 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
 
     l += __shfl_xor_sync(0xffffffffu, l, 1);
     l += __shfl_xor_sync(0xffffffffu, l, 2);
-    if (gq < G) {
-      const int h = item.kv_head * G + gq;
-      const int64_t slot = item.slot_base + static_cast<int64_t>(h) * item.n_slots + item.split;
+    const int64_t slot =
+        item.slot_base + static_cast<int64_t>(item.kv_head * G + (gq < G ? gq : 0)) * item.n_slots +
+        item.split;
+    const bool slot_ok = slot >= 0 && slot < a.part_slots;
+    if (!__all_sync(0xffffffffu, slot_ok || gq >= G) && lane == 0) atomicOr(a.status, kStatusBadSlot);
+    if (gq < G && slot_ok) {
       const float inv = 1.f / l;
       float* dst = a.part_o + slot * D;
 #pragma unroll

@@ -468,6 +468,35 @@ def test_out_of_pool_page_is_redirected_and_reported(mode):
     compare(out, lse, o_ref, l_ref, "after an out-of-pool page id")
 
 
+@pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
+def test_out_of_range_partial_slot_is_skipped_and_reported(mode):
+    # A plan whose first token's partial slots lie past the partial buffer
+    # (test hook): every kernel checks partial slots, so that token's
+    # partials are neither written nor read, the status word gets bit 16,
+    # the other tokens' outputs are exact and the next step is exact.
+    w = small_case(79, hq=8, hkv=2, d=128, prefix_len=[300, 40], req_agent=[0, 0, 1, 0],
+                   req_ctx=[10, 200, 33, 0], req_prefill=[0] * 4, req_decode=[1] * 4)
+    t, s = _session(w)
+    s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+    ids, q, kn, vn = s.decode_inputs()
+    lens = [s.ctx.query(B.Q_SUFFIX_LEN, r) for r in ids]
+    out, lse = s.new_outputs(len(ids))
+    out.fill_(3.0)
+    s.ctx.set_option(B.OPT_TEST_BAD_SLOT, 1)
+    s.decode(ids, q, kn, vn, out, lse)
+    assert s.ctx.device_status() == 16
+    ref = oracle.workload_decode(w, t)
+    assert torch.all(out[0].float() == 3.0)   # the skipped token's row was not written
+    o_ref, l_ref = stack_decode_ref(ref, range(1, len(ids)))
+    compare(out[1:], lse[1:], o_ref, l_ref, "other tokens beside a skipped slot")
+    s.ctx.request_truncate(ids, lens)
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(ref, range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "after an out-of-range partial slot")
+
+
 def test_plan_wait_timeout_is_reported_and_context_recovers():
     # A decode whose kernel never sees its plan (test hook: the flag it waits
     # for is never written) gives up at the device wait limit; the host reads
