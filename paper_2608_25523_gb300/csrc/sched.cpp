@@ -309,17 +309,43 @@ void Decider::run(tpa_sched_decision* out) {
   for (int a = 0; a < s_.n_agents; ++a)
     if (active_ >> a & 1) act.push_back(a);
   const int na = static_cast<int>(act.size());
-  auto repair = [&](Mask R) {
-    std::vector<Mask> sets;
+  // Single-agent edits of a prefix set (Sec. IV, the Repair neighbourhood):
+  // every drop, then every swap of a member for an active non-member.
+  auto add_repairs = [&](Mask R) {
     for (int a = 0; a < s_.n_agents; ++a)
-      if (R >> a & 1) sets.push_back(R & ~(Mask(1) << a));
+      if (R >> a & 1) add(R & ~(Mask(1) << a));
     for (int a = 0; a < s_.n_agents; ++a)
       if (R >> a & 1)
         for (int b : act)
-          if (!(R >> b & 1)) sets.push_back((R & ~(Mask(1) << a)) | (Mask(1) << b));
-    return sets;
+          if (!(R >> b & 1)) add((R & ~(Mask(1) << a)) | (Mask(1) << b));
+  };
+  // Every superset of R with `extra` (1 or 2) more active agents, in agent
+  // order; each adds its GreedyPack states.  Returns the best set's Phi and
+  // the set (the first one on ties), or -inf when R has no such superset.
+  auto best_superset = [&](Mask R, int extra, Mask* best_R) {
+    double best = kNegInf;
+    bool have = false;
+    auto consider = [&](Mask S) {
+      const double v = add(S);
+      if (!have || v > best) {
+        best = v;
+        *best_R = S;
+        have = true;
+      }
+    };
+    for (int x = 0; x < na; ++x) {
+      if (R >> act[x] & 1) continue;
+      if (extra == 1) {
+        consider(R | (Mask(1) << act[x]));
+        continue;
+      }
+      for (int y = x + 1; y < na; ++y)
+        if (!(R >> act[y] & 1)) consider(R | (Mask(1) << act[x]) | (Mask(1) << act[y]));
+    }
+    return have ? best : kNegInf;
   };
   if (na <= p_.M) {
+    // small pool: every prefix set of the active agents
     for (uint64_t mask = 0; mask < (uint64_t(1) << na); ++mask) {
       Mask R = 0;
       for (int j = 0; j < na; ++j)
@@ -327,9 +353,14 @@ void Decider::run(tpa_sched_decision* out) {
       add(R);
     }
   } else {
+    // large pool (Algorithm 1): a hill climb on Phi from the resident active
+    // prefixes.  It moves to the best one-agent superset while that raises
+    // Phi; where none does, it may take the best two-agent superset, once per
+    // decision; it stops when neither helps.  The start and the end point
+    // also contribute their Repair neighbourhoods, and the incumbent stays.
     Mask rg = r_now_ & active_;
     add(rg);
-    for (Mask R : repair(rg)) add(R);
+    add_repairs(rg);
     double phi_g;
     {
       std::vector<Cand> tmp;
@@ -338,51 +369,20 @@ void Decider::run(tpa_sched_decision* out) {
       for (const Cand& c : tmp)
         if (c.score > phi_g) phi_g = c.score;
     }
-    bool pair_tried = false;
-    while (true) {
-      double best_v = kNegInf;
-      Mask best_R = 0;
-      bool have = false;
-      for (int a : act) {
-        if (rg >> a & 1) continue;
-        const Mask R = rg | (Mask(1) << a);
-        const double v = add(R);
-        if (!have || v > best_v) {
-          best_v = v;
-          best_R = R;
-          have = true;
-        }
+    int two_agent_steps = 1;
+    for (;;) {
+      Mask next = 0;
+      double v = best_superset(rg, 1, &next);
+      if (!(v > phi_g)) {
+        if (two_agent_steps == 0) break;
+        --two_agent_steps;
+        v = best_superset(rg, 2, &next);
+        if (!(v > phi_g)) break;
       }
-      if (have && best_v > phi_g) {
-        rg = best_R;
-        phi_g = best_v;
-        continue;
-      }
-      if (pair_tried) break;
-      pair_tried = true;
-      std::vector<int> rest;
-      for (int a : act)
-        if (!(rg >> a & 1)) rest.push_back(a);
-      best_v = kNegInf;
-      have = false;
-      for (size_t x = 0; x < rest.size(); ++x)
-        for (size_t y = x + 1; y < rest.size(); ++y) {
-          const Mask R = rg | (Mask(1) << rest[x]) | (Mask(1) << rest[y]);
-          const double v = add(R);
-          if (!have || v > best_v) {
-            best_v = v;
-            best_R = R;
-            have = true;
-          }
-        }
-      if (have && best_v > phi_g) {
-        rg = best_R;
-        phi_g = best_v;
-      } else {
-        break;
-      }
+      rg = next;
+      phi_g = v;
     }
-    for (Mask R : repair(rg)) add(R);
+    add_repairs(rg);
     Cand inc;
     inc.agents = r_now_;
     inc.keep = running_;
