@@ -123,7 +123,7 @@ __device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) 
   SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, nullptr, p.n_sitems,
               p.stoks, p.full_prefix, p.tail_order, p.n_stok, p.n_full, p.split_keys, p.pages,
               p.squeue, p.status, p.num_pages, p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new,
-              p.k_pool, p.v_pool, p.part_slots};
+              p.k_pool, p.v_pool, p.part_slots, 1};
   split_warp_loop<D, G, kSplitStages>(a, ring, bars, abort_flag, lane);
 }
 

@@ -55,6 +55,8 @@ struct SplitArgs {
   __nv_bfloat16* k_pool;
   __nv_bfloat16* v_pool;
   int64_t part_slots;  // entries of part_lse; a slot outside [0, part_slots) is not written
+  int read_once;       // 1: every page is read by this launch once (request suffixes): its loads
+                       // are marked L2 evict-first, so the partials written meanwhile stay in L2
 };
 
 template <int D, int S>
@@ -178,8 +180,14 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
       const int z = static_cast<int>(pid * a.hkv + w.item.kv_head);
       fence_proxy_async();
       mbar_arrive_expect_tx(&bars[st], 2 * C::kPageBytes);
-      tma_load_5d(kst, a.tmap_k, &bars[st], 0, 0, 0, 0, z);
-      tma_load_5d(vst, a.tmap_v, &bars[st], 0, 0, 0, 0, z);
+      if (a.read_once) {
+        const uint64_t pol = l2_policy_evict_first();
+        tma_load_5d_hint(kst, a.tmap_k, &bars[st], 0, 0, 0, 0, z, pol);
+        tma_load_5d_hint(vst, a.tmap_v, &bars[st], 0, 0, 0, 0, z, pol);
+      } else {
+        tma_load_5d(kst, a.tmap_k, &bars[st], 0, 0, 0, 0, z);
+        tma_load_5d(vst, a.tmap_v, &bars[st], 0, 0, 0, 0, z);
+      }
     }
     ++issued;
   };
