@@ -1377,7 +1377,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
         CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
                               ctx->part_slots, ctx->status,
                               static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, ctx->num_sms,
-                              true, s));
+                              true, nullptr, 0, s));
       }
       launches = 3;
     } else {
@@ -1415,7 +1415,7 @@ int tpa_decode(tpa_ctx* ctx, int32_t n, const int32_t* reqs, const void* q, cons
         CUDA_TRY(launch_merge(dev_ptr<MergeTok>(sl, lay.off_merge), n, ctx->part_o, ctx->part_lse,
                               ctx->part_slots, ctx->status,
                               static_cast<__nv_bfloat16*>(out), lse, hq, ctx->d, ctx->num_sms,
-                              true, s));
+                              true, dp.plan_flag, dp.plan_seq, s));
       }
       launches = 2;
     }

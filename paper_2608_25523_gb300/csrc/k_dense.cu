@@ -97,8 +97,10 @@ enum { B_KFULL = 0, B_KEMPTY = 3, B_VFULL = 6, B_VEMPTY = 9, B_SFULL = 12, B_SFR
 // Split-KV role of a CTA of the same launch: 8 independent warps, each with
 // a 3-stage TMA page ring in the shared memory the dense role would use.
 
+// first: the CTA starts here (its programmatic-dependency wait is still to
+// come); otherwise it joins after its dense items, having waited already.
 template <int D, int G>
-__device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) {
+__device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem, bool first) {
   using W = SplitCfg<D, kSplitStages>;
   static_assert(kSplitWarps * (W::kWarpBytes + kSplitStages * 8) + 16 <= DenseCfg<D>::kSmem - 1024,
                 "split-KV rings fit in the launch's shared memory");
@@ -119,12 +121,13 @@ __device__ __forceinline__ void split_role(const DenseParams& p, uint8_t* smem) 
     prefetch_tmap(&p.tmap_k);
     prefetch_tmap(&p.tmap_v);
   }
-  pdl_wait();  // no global memory was touched before this point
+  // the wait for the kernel before this one comes inside the warp loop, once
+  // the first item is resolved from the plan (which no earlier kernel writes)
   SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, nullptr, p.n_sitems,
               p.stoks, p.full_prefix, p.tail_order, p.n_stok, p.n_full, p.split_keys, p.pages,
               p.squeue, p.status, p.num_pages, p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new,
               p.k_pool, p.v_pool, p.part_slots, 1};
-  split_warp_loop<D, G, kSplitStages>(a, ring, bars, abort_flag, lane);
+  split_warp_loop<D, G, kSplitStages>(a, ring, bars, abort_flag, lane, first);
 }
 
 template <int D, int G>
@@ -148,7 +151,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
     }
   }
   if (static_cast<int>(blockIdx.x) >= p.n_dense_ctas) {
-    split_role<D, G>(p, smem);
+    split_role<D, G>(p, smem, true);
     return;
   }
   const int warp = threadIdx.x >> 5;
@@ -570,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
   // consumed), so its warps join the split-KV work on the same shared memory.
   if (p.n_sitems > 0) {
     __syncthreads();
-    if (!*abort_flag) split_role<D, G>(p, smem);
+    if (!*abort_flag) split_role<D, G>(p, smem, false);
   }
 }
 

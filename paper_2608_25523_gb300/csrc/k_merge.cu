@@ -26,19 +26,33 @@ template <int D>
 __global__ void __launch_bounds__(kMergeThreads)
     merge_kernel(const MergeTok* __restrict__ toks, int n_tok, const float* __restrict__ part_o,
                  const float* __restrict__ part_lse, int64_t part_slots, uint32_t* status,
-                 __nv_bfloat16* __restrict__ out, float* __restrict__ lse_out, int hq) {
+                 __nv_bfloat16* __restrict__ out, float* __restrict__ lse_out, int hq,
+                 const unsigned long long* plan_flag, unsigned long long plan_seq) {
   pdl_trigger();  // the next step's main kernel may become resident now
-  pdl_wait();     // no-op unless launched as a dependent
   constexpr int LPI = D / 4;     // lanes per (token, head)
   constexpr int IPW = 32 / LPI;  // (token, head) pairs per warp and pass
   const int lane = threadIdx.x & 31;
   const int64_t total = static_cast<int64_t>(n_tok) * hq;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
-  for (int64_t w = warp * IPW + lane / LPI; w < total; w += nwarps * IPW) {
+  const int64_t w0 = warp * IPW + lane / LPI;
+  // With the plan uploaded ahead (its flag given), the first token record
+  // comes from the plan before waiting for the kernel that writes the
+  // partials; the partials are read after that wait.
+  MergeTok m0{0, 0, 0, 0};
+  if (plan_flag) {
+    const int got = threadIdx.x == 0 ? wait_flag64(plan_flag, plan_seq) : 1;
+    if (!__syncthreads_and(got)) {
+      if (threadIdx.x == 0) atomicOr(status, kStatusPlanTimeout);
+      return;
+    }
+    if (w0 < total) m0 = toks[w0 / hq];
+  }
+  pdl_wait();     // no-op unless launched as a dependent
+  for (int64_t w = w0; w < total; w += nwarps * IPW) {
     const int t = static_cast<int>(w / hq);
     const int h = static_cast<int>(w % hq);
-    const MergeTok m = toks[t];
+    const MergeTok m = (plan_flag && w == w0) ? m0 : toks[t];
     const int64_t base = m.slot_base + static_cast<int64_t>(h) * m.n_slots;
     const int col = 4 * (lane % LPI);
     if (base < 0 || m.n_slots < 0 || base + m.n_slots > part_slots) {
@@ -63,6 +77,7 @@ template <int D>
 cudaError_t launch_merge_t(const MergeTok* toks, int n_tok, const float* part_o,
                            const float* part_lse, int64_t part_slots, uint32_t* status,
                            __nv_bfloat16* out, float* lse, int hq, int num_sms, bool dependent,
+                           const unsigned long long* plan_flag, unsigned long long plan_seq,
                            cudaStream_t stream) {
   constexpr int IPB = (kMergeThreads / 32) * (32 / (D / 4));  // pairs per block and pass
   const int64_t pairs = static_cast<int64_t>(n_tok) * hq;
@@ -80,7 +95,7 @@ cudaError_t launch_merge_t(const MergeTok* toks, int n_tok, const float* part_o,
   cfg.attrs = attr;
   cfg.numAttrs = dependent ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, merge_kernel<D>, toks, n_tok, part_o, part_lse, part_slots, status,
-                            out, lse, hq);
+                            out, lse, hq, plan_flag, plan_seq);
 }
 
 }  // namespace
@@ -88,14 +103,15 @@ cudaError_t launch_merge_t(const MergeTok* toks, int n_tok, const float* part_o,
 cudaError_t launch_merge(const MergeTok* toks, int n_tok, const float* part_o,
                          const float* part_lse, int64_t part_slots, uint32_t* status,
                          __nv_bfloat16* out, float* lse, int hq, int d, int num_sms,
-                         bool dependent, cudaStream_t stream) {
+                         bool dependent, const unsigned long long* plan_flag,
+                         unsigned long long plan_seq, cudaStream_t stream) {
   if (n_tok <= 0) return cudaSuccess;
   if (d == 128)
     return launch_merge_t<128>(toks, n_tok, part_o, part_lse, part_slots, status, out, lse, hq,
-                               num_sms, dependent, stream);
+                               num_sms, dependent, plan_flag, plan_seq, stream);
   if (d == 64)
     return launch_merge_t<64>(toks, n_tok, part_o, part_lse, part_slots, status, out, lse, hq,
-                              num_sms, dependent, stream);
+                              num_sms, dependent, plan_flag, plan_seq, stream);
   return cudaErrorInvalidValue;
 }
 

@@ -41,7 +41,7 @@ __global__ void __launch_bounds__(128) suffix_kernel(const __grid_constant__ Suf
   SplitArgs a{&p.tmap_k, &p.tmap_v, p.q, p.part_o, p.part_lse, p.items, p.n_items,
               nullptr, nullptr, nullptr, 0, 0, 0, p.pages, p.queue, p.status, p.num_pages,
               p.hq, p.hkv, p.scale_log2, p.k_new, p.v_new, p.k_pool, p.v_pool, p.part_slots, 0};
-  split_warp_loop<D, G, S>(a, ring, bars, &abort_flag, lane);
+  split_warp_loop<D, G, S>(a, ring, bars, &abort_flag, lane, false);
 }
 
 template <int D, int G>

@@ -116,10 +116,13 @@ cudaError_t launch_suffix(const SuffixParams& p, int num_sms, int head_dim, int 
 // dependent = true launches it as a programmatic dependent of the kernel
 // before it on the stream (which triggers early): its CTAs become resident
 // while that kernel still runs and start merging the moment it completes.
+// plan_flag (non-null when the plan was uploaded ahead with that flag):
+// the kernel reads its first token record before its programmatic wait.
 cudaError_t launch_merge(const MergeTok* toks, int n_tok, const float* part_o,
                          const float* part_lse, int64_t part_slots, uint32_t* status,
                          __nv_bfloat16* out, float* lse, int hq, int d, int num_sms,
-                         bool dependent, cudaStream_t stream);
+                         bool dependent, const unsigned long long* plan_flag,
+                         unsigned long long plan_seq, cudaStream_t stream);
 
 // Raise dynamic shared-memory limits of the kernels (once per device).
 cudaError_t init_kernels();

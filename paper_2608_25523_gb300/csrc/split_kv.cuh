@@ -119,11 +119,14 @@ __device__ __forceinline__ SuffixItem fetch_item(const SplitArgs& a, int idx) {
 }  // namespace split_detail
 
 // Runs work items until the queue is empty.  `ring` is this warp's S stages,
-// `bars` its S initialised mbarriers (count 1).  Returns false after a
-// timeout (status bit set, in-flight copies drained).
+// `bars` its S initialised mbarriers (count 1).  wait_prev: the launch is a
+// programmatic dependent whose wait (griddepcontrol.wait) this loop makes
+// once its first item is resolved from the plan, before touching anything
+// earlier kernels wrote.  Returns false after a timeout (status bit set,
+// in-flight copies drained).
 template <int D, int G, int S>
 __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bars,
-                                volatile int* abort_flag, int lane) {
+                                volatile int* abort_flag, int lane, bool wait_prev) {
   using namespace split_detail;
   using C = SplitCfg<D, S>;
   const int gq = lane >> 2;  // mma group: query row of this lane
@@ -138,11 +141,14 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
     int npg;
     int32_t pid0, pid1;
   };
-  auto load_work = [&](int idx, Work& w) {  // whole warp
+  // The item and its page ids (plan data only)
+  auto resolve_work = [&](int idx, Work& w) {  // whole warp
     w.item = fetch_item(a, idx);
     w.npg = (w.item.n_keys + kPage - 1) / kPage;
     w.pid0 = lane < w.npg ? __ldg(a.pages + w.item.pages + lane) : 0;
     w.pid1 = lane + 32 < w.npg ? __ldg(a.pages + w.item.pages + lane + 32) : 0;
+  };
+  auto append_work = [&](const Work& w) {  // whole warp
     if (w.item.app_src >= 0 && a.k_new) {
       // append the step's token to the pool before its page is loaded (its
       // page belongs to this item alone: key ranges start on page boundaries)
@@ -163,6 +169,10 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
       asm volatile("fence.proxy.async.global;" ::: "memory");
       __syncwarp();
     }
+  };
+  auto load_work = [&](int idx, Work& w) {
+    resolve_work(idx, w);
+    append_work(w);
   };
   // TMA page `pg` of `w` into ring slot issued % S (whole warp; lane 0 issues)
   auto issue = [&](const Work& w, int pg) {
@@ -193,11 +203,15 @@ __device__ bool split_warp_loop(const SplitArgs& a, uint8_t* ring, uint64_t* bar
   };
   auto claim = [&]() -> uint32_t { return lane == 0 ? atomicAdd(a.queue, 1u) : 0u; };
 
+  // The first item is claimed and resolved from the plan before waiting for
+  // the previous kernel (wait_prev); its append and page loads come after.
   int idx = __shfl_sync(0xffffffffu, static_cast<int>(claim()), 0);
   Work cur{};
   int cur_iss = 0;  // pages of cur issued
+  if (idx < a.n_items) resolve_work(idx, cur);
+  if (wait_prev) pdl_wait();
   if (idx < a.n_items) {
-    load_work(idx, cur);
+    append_work(cur);
     while (cur_iss < cur.npg && cur_iss < S) issue(cur, cur_iss++);
   }
 
