@@ -82,7 +82,19 @@ cudaError_t launch_merge_t(const MergeTok* toks, int n_tok, const float* part_o,
   constexpr int IPB = (kMergeThreads / 32) * (32 / (D / 4));  // pairs per block and pass
   const int64_t pairs = static_cast<int64_t>(n_tok) * hq;
   int64_t blocks = (pairs + IPB - 1) / IPB;
-  const int64_t cap = static_cast<int64_t>(num_sms > 0 ? num_sms : 1) * 8;
+  // At most one wave: as many blocks as can be resident at once (blocks
+  // beyond that would start only as the first ones finish and double the
+  // latency chain of the pairs they loop over).
+  static int per_sm = 0;
+  if (per_sm == 0) {
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, merge_kernel<D>, kMergeThreads, 0) !=
+            cudaSuccess ||
+        n < 1)
+      n = 1;
+    per_sm = n;
+  }
+  const int64_t cap = static_cast<int64_t>(num_sms > 0 ? num_sms : 1) * per_sm;
   if (blocks > cap) blocks = cap;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(blocks));
