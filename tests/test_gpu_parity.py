@@ -128,6 +128,56 @@ def test_decode_sharp_softmax():
     compare(out, lse, o_ref, l_ref, "sharp")
 
 
+@pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
+def test_decode_steps_back_to_back(mode):
+    """12 decode steps issued with no host synchronisation between them, each
+    appending one token per request and writing its own outputs: the steps
+    run as a chain of programmatic dependents (each step's split-KV warps
+    resolve their first item from the plan before waiting for the previous
+    kernel) and cycle the 4-slot plan ring three times.  Every step must
+    match the oracle."""
+    steps = 12
+    n = 6
+    w = small_case(83, hq=8, hkv=2, d=128, prefix_len=[700, 129, 0], req_agent=[0, 1, 0, 2, 1, 0],
+                   req_ctx=[0] * n, req_prefill=[40, 300, 17, 260, 1, 120],
+                   req_decode=[1] * n, chunk=512, permute=True)
+    t = tensors_numpy(w)
+    s = Session(w, to_device(t, "cuda"))
+    s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+    td = s.t
+    ids = list(range(n))
+    # prefill the inputs except their last `steps` tokens, which the decode steps append
+    base = [w.req_prefill[r] - steps if w.req_prefill[r] > steps else 0 for r in ids]
+    pre = [r for r in ids if base[r] > 0]
+    if pre:
+        q = torch.cat([td.q_prefill[td.qpf_off[r]:td.qpf_off[r] + base[r]] for r in pre])
+        kv = [td.suffix(r, w, 0, base[r]) for r in pre]
+        out, lse = s.new_outputs(sum(base[r] for r in pre))
+        s.prefill(pre, [base[r] for r in pre], q, torch.cat([k for k, _ in kv]),
+                  torch.cat([v for _, v in kv]), out, lse)
+    live = [r for r in ids if w.req_prefill[r] >= steps]   # requests with a token for every step
+    results = []
+    for j in range(steps):
+        pos = [base[r] + j for r in live]
+        q = torch.stack([td.q_prefill[td.qpf_off[r] + p] for r, p in zip(live, pos)])
+        kn = torch.stack([td.suffix(r, w, p, p + 1)[0][0] for r, p in zip(live, pos)])
+        vn = torch.stack([td.suffix(r, w, p, p + 1)[1][0] for r, p in zip(live, pos)])
+        out, lse = s.new_outputs(len(live))
+        s.decode(live, q, kn, vn, out, lse)
+        results.append((pos, q, out, lse))
+    torch.cuda.synchronize()
+    _check_status(s)
+    for j, (pos, q, out, lse) in enumerate(results):
+        refs = []
+        for r, p, qr in zip(live, pos, q):
+            pk, pv = t.prefix(w.req_agent[r], w)
+            sk, sv = t.suffix(r, w, 0, p)
+            nk, nv = t.suffix(r, w, p, p + 1)
+            refs.append(oracle.decode_step(qr.float().cpu().numpy(), pk, pv, sk, sv, nk[0], nv[0]))
+        compare(out, lse, np.stack([o for o, _ in refs]), np.stack([l for _, l in refs]),
+                f"back-to-back step {j}")
+
+
 def test_cascade_equals_flat():
     """The two-level cascade and the flat split-KV path read the same keys
     in different groupings; they agree to fp32 reordering noise."""
