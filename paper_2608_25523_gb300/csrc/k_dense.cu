@@ -34,7 +34,8 @@
 //   warps 2..9  warp w owns TMEM lane quarter w % 4 (rows 32(w%4)..+31) and
 //               key half (w-2)/4.  Per tile: read S, take the full-row max
 //               (both warps of a pair, so their running max agrees without
-//               synchronising), write P (bf16) for their key half into
+//               synchronising; the load-with-maximum form of tcgen05.ld
+//               gives it for a full tile), write P (bf16) for their key half into
 //               TMEM, rescale O in
 //               TMEM only when the max grew by more than 2^8 (otherwise the
 //               stale max stays the reference, which is exact: it is only a
@@ -385,11 +386,13 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
         }
         tc_fence_after();
         const uint32_t scol = tmem + lane_base + (s ? C::kColS1 : C::kColS0);
-        float x[64], y[64];
-        tmem_ld32(scol + own, x);
-        tmem_ld32(scol + own + 32, x + 32);
-        tmem_ld32(scol + other, y);
-        tmem_ld32(scol + other + 32, y + 32);
+        // both key halves of the row, each 32 columns with its maximum taken
+        // by the TMEM load itself
+        float x[64], y[64], cmax[4];
+        tmem_ld32_max(scol + own, x, cmax[0]);
+        tmem_ld32_max(scol + own + 32, x + 32, cmax[1]);
+        tmem_ld32_max(scol + other, y, cmax[2]);
+        tmem_ld32_max(scol + other + 32, y + 32, cmax[3]);
         tmem_wait_ld();
         tc_fence_before();
         mbar_arrive(&bars[B_SFREE + s]);
@@ -399,25 +402,27 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(const __grid_constan
           const int c = dt.causal_pos - t.key0 + 1;
           lim = c > 0 ? c : 0;
         }
+        float mraw = fmaxf(fmax3f(cmax[0], cmax[1], cmax[2]), cmax[3]);
         if (lim < 128) {
+          // keys past the range or the causal limit: masked, and the full-row
+          // max taken again over the keys that remain (8 chains of 3-input max)
 #pragma unroll
           for (int n = 0; n < 64; ++n) {
             x[n] = own + n < lim ? x[n] : -INFINITY;
             y[n] = other + n < lim ? y[n] : -INFINITY;
           }
+          float acc[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) acc[i] = fmax3f(x[i], x[i + 8], y[i]);
+#pragma unroll
+          for (int kk = 16; kk < 64; kk += 8)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], x[kk + i], y[kk + i - 8]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) acc[i] = fmaxf(acc[i], y[56 + i]);
+          mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
+                        fmaxf(acc[6], acc[7]));
         }
-        // full-row max of the raw scores: 8 independent chains of 3-input max
-        float acc[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = fmax3f(x[i], x[i + 8], y[i]);
-#pragma unroll
-        for (int kk = 16; kk < 64; kk += 8)
-#pragma unroll
-          for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], x[kk + i], y[kk + i - 8]);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = fmaxf(acc[i], y[56 + i]);
-        const float mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
-                                  fmaxf(acc[6], acc[7]));
         const float mx = mraw * sc;  // sc > 0: max of the scaled scores
         const float m_new = fmaxf(m_run, mx);
         const bool grow = m_new > m_run + kRescaleThreshold;

@@ -28,7 +28,9 @@
 //               PV_X(j) has read it.
 //   softmax     warp w owns TMEM lane quarter w % 4 and each thread one
 //               query row of its tile (a whole warpgroup per tile), all 128
-//               keys of a tile: read S, row max, P = 2^(s - m) as bf16 into
+//               keys of a tile: read S (the load-with-maximum form of
+//               tcgen05.ld gives the row max of a full tile; a ragged or
+//               causal tile takes it again after masking), P = 2^(s - m) as bf16 into
 //               the first 64 columns of its S buffer, row sum; O is rescaled
 //               in TMEM only when the max grew by more than 2^8 (the stale max
 //               stays the reference otherwise, which is exact: it is only a
@@ -319,9 +321,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
         const int g = gt + j;
         if (!wait_all(sfull, g & 1)) break;
         tc_fence_after();
-        float s[128];
+        // S with the maximum of each 32 columns, taken by the TMEM load itself
+        float s[128], cmax[4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(scol + 32 * c, s + 32 * c);
+        for (int c = 0; c < 4; ++c) tmem_ld32_max(scol + 32 * c, s + 32 * c, cmax[c]);
         tmem_wait_ld();
 
         int lim = t.nvalid;
@@ -329,20 +332,22 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_pair_kernel(const __grid_
           const int c = dt.causal_pos - t.key0 + 1;
           lim = c > 0 ? c : 0;
         }
+        float mraw = fmaxf(fmax3f(cmax[0], cmax[1], cmax[2]), cmax[3]);
         if (lim < 128) {
+          // keys past the range or the causal limit: masked, and the row max
+          // taken again over the keys that remain (8 chains of 3-input max)
 #pragma unroll
           for (int n = 0; n < 128; ++n) s[n] = n < lim ? s[n] : -INFINITY;
+          float acc[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) acc[i] = s[i];
+#pragma unroll
+          for (int kk = 8; kk < 128; kk += 16)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], s[kk + i], s[kk + 8 + i]);
+          mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
+                        fmaxf(acc[6], acc[7]));
         }
-        // row max of the raw scores: 8 independent chains of 3-input max
-        float acc[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = s[i];
-#pragma unroll
-        for (int kk = 8; kk < 128; kk += 16)
-#pragma unroll
-          for (int i = 0; i < 8; ++i) acc[i] = fmax3f(acc[i], s[kk + i], s[kk + 8 + i]);
-        const float mraw = fmax3f(fmax3f(acc[0], acc[1], acc[2]), fmax3f(acc[3], acc[4], acc[5]),
-                                  fmaxf(acc[6], acc[7]));
         const float mx = mraw * sc;  // sc > 0: max of the scaled scores
         const float m_new = fmaxf(m_run, mx);
         const bool grow = m_new > m_run + kRescaleThreshold;
