@@ -622,6 +622,7 @@ def bench_prefill(args, dev, tf_peak, peak_src):
             "roofline": {"bound": "tensor", "kernel": kname, "achieved": round(ach, 1),
                          "peak": tf_peak, "unit": "TFLOP/s", "frac": round(ach / tf_peak, 4),
                          "peak_source": peak_src, "traffic": None,
+                         "frac_of_sustained": round(ach / peaks()[2], 4),
                          "avg_launch_us": round(1e3 * dense_ms / max(1, kt[kname][1]), 1)},
             "device_status": st}
 
@@ -1135,6 +1136,7 @@ def compact(res):
     if x:
         out["decode_8b"] = {"value": x["value"], "unit": "GB/s", "steps": x["steps"],
                             "ms_per_step": x["ms_per_step"], "frac": x["roofline"]["frac"],
+                            "frac_of_8tbs": x.get("hbm_frac_of_8tbs"),
                             "bracketed_kernel_us": x["roofline"]["bracketed_avg_us"],
                             "steps20_ms_per_step": x["steps20_ms_per_step"],
                             "tokens_per_s": x["tokens_per_s"], "e2e_gbs": x["e2e"]["value"],
@@ -1143,7 +1145,9 @@ def compact(res):
     if x:
         out["prefill"] = {"tflops": x["tflops"], "ms": x["ms"], "tokens_per_s": x["tokens_per_s"],
                           "kernel_tflops": x["roofline"]["achieved"], "frac": x["roofline"]["frac"],
-                          "peak": x["roofline"]["peak"], "device_status": x["device_status"]}
+                          "peak": x["roofline"]["peak"],
+                          "frac_of_sustained": x["roofline"].get("frac_of_sustained"),
+                          "device_status": x["device_status"]}
     x = res.get("mixed")
     if x:
         k = x["kernels_per_step"]
