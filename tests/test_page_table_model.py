@@ -320,6 +320,7 @@ class PageTableMachine(RuleBasedStateMachine):
             assert suffixes[r] == (self.suffix[r][1] if r in self.suffix else -1), r
 
 
-PageTableMachine.TestCase.settings = settings(max_examples=200, stateful_step_count=40,
+PageTableMachine.TestCase.settings = settings(max_examples=300, stateful_step_count=40,
+                                              derandomize=True, database=None,
                                               deadline=None)
 test_page_tables = PageTableMachine.TestCase
