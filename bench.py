@@ -835,8 +835,18 @@ def bench_movement(args, dev):
             exact = bool(torch.equal(ok[:ell].view(torch.int16), hk[:ell].view(torch.int16)) and
                          torch.equal(ov[:ell].view(torch.int16), hv[:ell].view(torch.int16)))
             t_h2d, t_d2h = timed(h2d), timed(d2h)
+            # the staged reload's page scatter alone (its kernel bracketed by events):
+            # it reads the staging area and writes the pages, 2 x bytes of HBM traffic
+            ctx.set_option(B.OPT_KERNEL_TIMING, 1)
+            ctx.kernel_times(reset=True)
+            timed(reload, before=evict)
+            kt = ctx.kernel_times(reset=True)
+            ctx.set_option(B.OPT_KERNEL_TIMING, 0)
+            scatter_us = 1e3 * kt["page_copy"][0] / max(1, kt["page_copy"][1])
         side.synchronize()
         rows.append({"tokens": ell, "bytes": ell * mu, "reload_us": round(t_re, 1),
+                     "scatter_kernel_us": round(scatter_us, 1),
+                     "scatter_hbm_gbs": round(2 * ell * mu / (scatter_us * 1e-6) / 1e9, 1),
                      "offload_us": round(t_off, 1), "reload_direct_us": round(t_re_d, 1),
                      "offload_direct_us": round(t_off_d, 1), "h2d_copy_us": round(t_h2d, 1),
                      "d2h_copy_us": round(t_d2h, 1), "round_trip_bit_exact": exact})
@@ -856,6 +866,13 @@ def bench_movement(args, dev):
            "rows": rows, "reload": fit("reload_us"), "offload": fit("offload_us"),
            "reload_direct": fit("reload_direct_us"), "offload_direct": fit("offload_direct_us"),
            "h2d_copy": fit("h2d_copy_us"), "d2h_copy": fit("d2h_copy_us")}
+    big = rows[-1]
+    hbm_peak = peaks()[0]
+    res["reload_scatter"] = {
+        "tokens": big["tokens"], "kernel_us": big["scatter_kernel_us"],
+        "hbm_gbs": big["scatter_hbm_gbs"], "frac": round(big["scatter_hbm_gbs"] / hbm_peak, 4),
+        "frac_of_8tbs": round(big["scatter_hbm_gbs"] / 8000.0, 4),
+        "bytes": "staging area read + pages written, 2 x the prefix's bytes"}
     res["mu_over_B_swap_ns_per_token"] = {
         "reload": round(mu / (res["reload"]["B_gbs"] * 1e9) * 1e9, 3),
         "offload": round(mu / (res["offload"]["B_gbs"] * 1e9) * 1e9, 3)}
@@ -1163,6 +1180,8 @@ def compact(res):
                            "offload_direct_gbs": x["offload_direct"]["B_gbs"],
                            "h2d_copy_gbs": x["h2d_copy"]["B_gbs"],
                            "mu_over_B_swap_ns": x["mu_over_B_swap_ns_per_token"]["reload"],
+                           "reload_scatter_hbm_gbs": (x.get("reload_scatter") or {}).get("hbm_gbs"),
+                           "reload_scatter_frac": (x.get("reload_scatter") or {}).get("frac"),
                            "bit_exact": all(r["round_trip_bit_exact"] for r in x["rows"])}
     x = res.get("redo")
     if x:
