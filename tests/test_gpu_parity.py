@@ -95,6 +95,40 @@ def test_decode_split_choices_agree(splits):
 
 
 @pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
+def test_decode_at_capacity_limits(mode):
+    """A batch of exactly max_tokens requests whose suffixes reach
+    max_seq_len with the step's token, under a split budget (max_splits 4)
+    so small that the planner must widen the suffix items: every row matches
+    the oracle.  The next step would pass max_seq_len and is refused with
+    CAPACITY, with the tables left as they were."""
+    n = 48
+    ctx_lens = [1599 if i % 5 == 0 else (37 * i) % 1599 for i in range(n)]
+    w = small_case(61, hq=8, hkv=2, d=128, prefix_len=[100, 1], req_agent=[i % 2 for i in range(n)],
+                   req_ctx=ctx_lens, req_prefill=[0] * n, req_decode=[1] * n, permute=True)
+    t = tensors_numpy(w)
+    s = Session(w, to_device(t, "cuda"), extra_tokens=0, max_splits=4, max_tokens=n)
+    s.ctx.set_option(B.OPT_DECODE_MODE, mode)
+    ids, q, kn, vn = s.decode_inputs()
+    assert len(ids) == n
+    out, lse = s.new_outputs(n)
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(n))
+    compare(out, lse, o_ref, l_ref, f"capacity limits/{mode}")
+    lens = [s.ctx.query(B.Q_SUFFIX_LEN, r) for r in ids]
+    assert max(lens) == 1600
+    free = s.ctx.query(B.Q_FREE_PAGES)
+    with pytest.raises(B.TpaError) as e:
+        s.decode(ids, q, kn, vn, out, lse)
+    assert e.value.code == B.TPA_ERR_CAPACITY
+    assert [s.ctx.query(B.Q_SUFFIX_LEN, r) for r in ids] == lens
+    assert s.ctx.query(B.Q_FREE_PAGES) == free
+    torch.cuda.synchronize()
+    _check_status(s)
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
 def test_decode_suffix_scores_far_above_the_prefix(mode):
     """Suffix keys 24x larger than the prefix keys: the partials of one
     token have LSEs tens of units apart, so the exact merge must weight the
