@@ -289,6 +289,41 @@ def test_prefill_scores_rising_far_above_the_first_tile(rows):
         row += c
 
 
+@pytest.mark.parametrize("rows", [256, 128], ids=["pairs", "single"])
+def test_prefill_at_capacity_limits(rows):
+    """One call whose chunks total exactly max_tokens rows, one of them
+    ending exactly at max_seq_len (cached suffixes before the chunks): every
+    row matches the oracle.  One more token for that request is refused
+    with CAPACITY, with the tables left as they were."""
+    w = small_case(67, hq=8, hkv=2, d=128, prefix_len=[150, 17], req_agent=[0, 1, 0, 1],
+                   req_ctx=[0, 40, 100, 7], req_prefill=[200, 150, 90, 200], req_decode=[0] * 4,
+                   chunk=256, permute=True)
+    t = tensors_numpy(w)
+    s = Session(w, to_device(t, "cuda"), extra_tokens=0, max_tokens=640)
+    s.ctx.set_option(B.OPT_PREFILL_TILE_ROWS, rows)
+    assert w.prefill_rounds() == 1
+    chunks, ids, lens, q, k, v = s.prefill_inputs(0)
+    assert sum(lens) == 640
+    out, lse = s.new_outputs(640)
+    s.prefill(ids, lens, q, k, v, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    row = 0
+    for r, off, c in chunks:
+        o_ref, l_ref = oracle.workload_prefill_chunk(w, t, r, off, c)
+        compare(out[row:row + c], lse[row:row + c], o_ref, l_ref, f"capacity r{r} off{off}")
+        row += c
+    assert s.ctx.query(B.Q_SUFFIX_LEN, 3) == 207
+    free = s.ctx.query(B.Q_FREE_PAGES)
+    with pytest.raises(B.TpaError) as e:
+        s.prefill([3], [1], q[:1], k[:1], v[:1], out[:1], lse[:1])
+    assert e.value.code == B.TPA_ERR_CAPACITY
+    assert s.ctx.query(B.Q_SUFFIX_LEN, 3) == 207
+    assert s.ctx.query(B.Q_FREE_PAGES) == free
+    torch.cuda.synchronize()
+    _check_status(s)
+
+
 def test_tiny_workload_prefill_then_decode():
     """The tiny workload: 1 agent, 256-token prefix, 4 requests prefill a
     64-token suffix in one chunk, then take one decode step."""
