@@ -552,15 +552,31 @@ def test_prefill_runs_ready_chunks_before_a_pending_reload(rows, only_reloading)
 
 
 def test_reload_rejects_unpinned_host_memory():
+    """A reload that fails (pageable host memory) leaves the prefix evicted:
+    the agent's decode is refused with NOT_RESIDENT rather than waiting, and
+    after a good reload (pinned copies of the prefix) the step is exact."""
     w = small_case(25, hq=8, hkv=2, d=64, prefix_len=[40], req_agent=[0], req_ctx=[1],
                    req_prefill=[0], req_decode=[1])
     t, s = _session(w)
+    pk, pv = s.t.prefix(0, w)
+    hk_good, hv_good = pk.cpu().pin_memory(), pv.cpu().pin_memory()
     s.ctx.prefix_evict(0)
     hk = torch.zeros(40, 2, 64, dtype=torch.bfloat16)   # pageable
     with pytest.raises(B.TpaError) as e:
         s.ctx.prefix_reload(0, hk, hk)
     assert e.value.code == B.TPA_ERR_INVALID_ARG
     assert s.ctx.query(B.Q_PREFIX_RESIDENT, 0) == 0
+    ids, q, kn, vn = s.decode_inputs()
+    out, lse = s.new_outputs(len(ids))
+    with pytest.raises(B.TpaError) as e:
+        s.decode(ids, q, kn, vn, out, lse)
+    assert e.value.code == B.TPA_ERR_NOT_RESIDENT
+    s.ctx.prefix_reload(0, hk_good, hv_good)
+    s.decode(ids, q, kn, vn, out, lse)
+    torch.cuda.synchronize()
+    _check_status(s)
+    o_ref, l_ref = stack_decode_ref(oracle.workload_decode(w, t), range(len(ids)))
+    compare(out, lse, o_ref, l_ref, "after a failed and a good reload")
 
 
 @pytest.mark.parametrize("mode", [0, 1], ids=["cascade", "flat"])
